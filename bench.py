@@ -1,0 +1,368 @@
+"""Throughput of the Sparse-Reslim routed encoder forward on GB300.
+
+One step = one sr_forward over one batch of the 0.25 degree workload (B = 1,
+720x1440 grid, patch 8 -> L = 16200 tokens, D = 1024, 16 heads, 24 blocks
+split (4, 16, 4), keep ratio 0.25 -> K = 4050 routed tokens, bf16 storage,
+fp32 accumulation), inputs resident in HBM.  Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the fp64 CPU oracle on the host cores
+
+Multi-GPU (torchrun): every rank runs an independent replica on its own batch
+(the forward has no cross-sample exchange), so scaling is weak.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "c4_0p25deg_bf16"
+L2_FLUSH_BYTES = 512 << 20          # > 129 MB of L2
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": p["hbm_gbs"], "bf16_tflops": p["bf16_tflops"],
+                "bf16_tflops_sustained": p["bf16_tflops_sustained"], "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+def _workload(name):
+    from paper_2607_02829_gb300 import synth
+    if name in synth.WORKLOADS:
+        return synth.WORKLOADS[name]
+    for wl in synth.sweep_workloads():
+        if wl.name == name:
+            return wl
+    raise SystemExit(f"unknown workload {name}")
+
+
+def _describe(wl, K):
+    return {"workload": wl.name, "grid": f"{wl.grid_h}x{wl.grid_w}", "channels": wl.channels,
+            "patch": wl.patch, "B": wl.B, "L": wl.L, "D": wl.D, "heads": wl.heads,
+            "split": [wl.n1, wl.n2, wl.n3], "keep_ratio": wl.keep_ratio, "K": K,
+            "selector": wl.selector, "storage": wl.dtype}
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason sampling during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+            self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                p = [v.strip() for v in line.split(",")]
+                if len(p) < 9:
+                    continue
+                try:
+                    sm.append(float(p[1]))
+                    smax = float(p[2])
+                except ValueError:
+                    continue
+                for n, v in zip(names, p[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        if not sm:
+            return None
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+    from paper_2607_02829_gb300 import binding as b, synth
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    wl = _workload(args.workload)
+    K = b.sr_keep_count(wl.L, wl.keep_ratio)
+    cfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, wl.n1, wl.n2, wl.n3, dtype=wl.dtype,
+                        selector=wl.selector)
+    enc = b.Encoder(cfg, max_keep_ratio=wl.keep_ratio)
+    # each rank: its own batch (seeded by rank), shared weights
+    x_cpu, w_cpu = synth.make_inputs(wl.with_(seed_index=wl.seed_index + 100 * rank)
+                                     if rank else wl)
+    x = x_cpu.to(dev)
+    wd = [{k: v.to(dev) for k, v in blk.items()} for blk in w_cpu]
+    warr = b.weights_array(wd)
+    out = torch.empty_like(x)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    seed = wl.select_seed
+
+    def step(i):
+        b.sr_forward(enc.handle, x.data_ptr(), warr, wl.keep_ratio, seed + i, out.data_ptr(),
+                     None, stream.cuda_stream)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+
+    # ---- timed region: K steps, L2 flushed before each, events around each step
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        step(args.warmup + i)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    wall = time.perf_counter() - t0
+    clk = clocks.stop()
+    ms = sum(a.elapsed_time(z) for a, z in ev) / args.steps
+    ms_t = torch.tensor([ms], device=dev)
+    if world > 1:
+        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
+    ms = float(ms_t.item())
+
+    # ---- per-kernel trace over K more steps (same launches, events around each)
+    b.sr_trace_enable(enc.handle, True)
+    b.sr_trace_read(enc.handle, reset=True)
+    for i in range(args.steps):
+        flush.zero_()
+        step(args.warmup + i)
+    torch.cuda.synchronize()
+    trace = b.sr_trace_read(enc.handle, reset=True)
+    b.sr_trace_enable(enc.handle, False)
+
+    # ---- end to end through the C ABI from pinned host memory
+    xh = x_cpu.pin_memory()
+    oh = torch.empty_like(xh).pin_memory()
+    dbuf = torch.empty_like(x)
+    bytes_io = x.numel() * x.element_size()
+    for i in range(max(1, args.warmup // 2)):
+        b.sr_forward_host(enc.handle, xh.data_ptr(), warr, wl.keep_ratio, seed, dbuf.data_ptr(),
+                          oh.data_ptr(), None, stream.cuda_stream)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    e0.record(stream)
+    for i in range(args.steps):
+        b.sr_forward_host(enc.handle, xh.data_ptr(), warr, wl.keep_ratio, seed + i,
+                          dbuf.data_ptr(), oh.data_ptr(), None, stream.cuda_stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / args.steps
+    e2e_t = torch.tensor([e2e_ms], device=dev)
+    if world > 1:
+        dist.all_reduce(e2e_t, op=dist.ReduceOp.MAX)
+    e2e_ms = float(e2e_t.item())
+    enc.close()
+    return wl, K, ms, wall, clk, trace, e2e_ms, bytes_io
+
+
+def roofline(trace, peaks, steps):
+    kernels = {k: v for k, v in trace.items() if k != "copy" and v["launches"] > 0}
+    dom = max(kernels, key=lambda k: kernels[k]["ms"])
+    t = kernels[dom]
+    per_launch_ms = t["ms"] / t["launches"]
+    if t["flops"] > 0:
+        achieved = t["flops"] / t["launches"] / (per_launch_ms * 1e-3) / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        bound, unit = "tensor", "TFLOP/s"
+    else:
+        achieved = t["bytes"] / t["launches"] / (per_launch_ms * 1e-3) / 1e9
+        peak = peaks["hbm_gbs"]
+        bound, unit = "hbm", "GB/s"
+    total_ms = sum(v["ms"] for v in kernels.values())
+    detail = {}
+    for k, v in kernels.items():
+        d = {"launches_per_step": v["launches"] / steps, "ms_per_step": v["ms"] / steps,
+             "share": v["ms"] / total_ms}
+        if v["flops"] > 0:
+            d["tflops"] = v["flops"] / (v["ms"] * 1e-3) / 1e12
+        if v["bytes"] > 0:
+            d["gbs"] = v["bytes"] / (v["ms"] * 1e-3) / 1e9
+        detail[k] = d
+    return ({"kernel": dom, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+             "frac": achieved / peak, "peak_source": peaks["source"] +
+             (" sustained" if bound == "tensor" else ""), "traffic": None}, detail)
+
+
+def cpu_baseline(wl, budget_s=25.0):
+    """The fp64 oracle, as it stands, on a bounded sample of the workload: one dense
+    block over all L tokens and one sparse block over the K routed tokens of the
+    same model; the full forward's time is those block times weighted by the
+    block counts (selection and gather are negligible next to the blocks)."""
+    import numpy as np
+    from oracle import reslim as o
+    from paper_2607_02829_gb300 import synth
+    threads = len(os.sched_getaffinity(0))
+    rng = np.random.Generator(np.random.PCG64(7))
+    x = synth.stored_as_f64(synth.to_storage(synth.make_tokens(wl), wl.dtype))
+    w = o.as_f64_weights([{k: synth.to_storage(v, wl.dtype) for k, v in
+                           synth.make_block_weights(wl.D, wl.mlp_hidden, 1).items()}])[0]
+    K = o.keep_count(wl.L, wl.keep_ratio)
+    from concurrent.futures import ThreadPoolExecutor
+    pool = ThreadPoolExecutor(threads)
+    t0 = time.perf_counter()
+    o.block(x, w, wl.heads, pool=pool)
+    t_dense = time.perf_counter() - t0
+    idx = o.select_random(wl.B, wl.L, K, 1)
+    h = x[np.arange(wl.B)[:, None], idx]
+    t0 = time.perf_counter()
+    o.block(h, w, wl.heads, pool=pool)
+    t_sparse = time.perf_counter() - t0
+    pool.shutdown()
+    n_dense = wl.n1 + wl.n3 + (wl.n2 if wl.keep_ratio == 1.0 else 0)
+    n_sparse = 0 if wl.keep_ratio == 1.0 else wl.n2
+    est = n_dense * t_dense + n_sparse * t_sparse
+    return {"value": wl.B * wl.L / est, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+            "sample": f"one dense block (T={wl.L}) + one sparse block (T={K}) of {wl.name}, "
+                      f"{t_dense:.1f} s + {t_sparse:.1f} s fp64, weighted by {n_dense} dense "
+                      f"+ {n_sparse} sparse blocks -> {est:.0f} s per forward",
+            "sample_seconds": t_dense + t_sparse}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+
+    import torch
+    import torch.distributed as dist
+    if world > 1:
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    # build once per node, then every rank loads the library
+    if local_rank == 0:
+        from paper_2607_02829_gb300 import build
+        build.build()
+    if world > 1:
+        dist.barrier()
+
+    wl, K, ms, wall, clk, trace, e2e_ms, bytes_io = run_ours(args, rank, world, local_rank)
+    peaks = _peaks()
+    tokens = wl.B * wl.L * world
+    value = tokens / (ms * 1e-3)
+    roof, detail = roofline(trace, peaks, args.steps)
+    launches = sum(v["launches"] for k, v in trace.items() if k != "copy")
+    gs = {}
+    for k in ("gather", "gemm_fc2_scatter"):
+        if trace[k]["launches"]:
+            gs[k + "_gbs"] = trace[k]["bytes"] / (trace[k]["ms"] * 1e-3) / 1e9
+    total_flops = sum(v["flops"] for v in trace.values()) / args.steps
+    line = {
+        "metric": "full-grid tokens/sec of routed encoder fwd",
+        "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
+        "data": "synthetic (seeded ERA5-shaped smooth fields, random-init weights)",
+        "config": dict(_describe(wl, K), l2="flushed (512 MB write) before every timed step",
+                       parallelism=f"replicas x{world}"),
+        "roofline": roof,
+        "forward_tflops": total_flops / (ms * 1e-3) / 1e12,
+        "gather_scatter": gs,
+        "kernels": detail,
+        "e2e": {"value": tokens / (e2e_ms * 1e-3), "unit": "tokens/s",
+                "h2d_bytes_per_step": bytes_io, "d2h_bytes_per_step": bytes_io},
+        "gpu_launches": int(launches),
+        "wall_s_timed_region": wall,
+        "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_reference(args, rank, world):
+    """The oracle as the reference arm, on the host cores, rank 0 only."""
+    if rank != 0:
+        return
+    wl = _workload(args.workload)
+    from oracle import reslim as o
+    K = o.keep_count(wl.L, wl.keep_ratio)
+    vals = []
+    base = None
+    for i in range(args.warmup + args.steps):
+        base = cpu_baseline(wl)
+        if i >= args.warmup:
+            vals.append(base["value"])
+    value = sum(vals) / len(vals)
+    ms = wl.B * wl.L / value * 1e3
+    line = {"impl": "reference", "metric": "full-grid tokens/sec of routed encoder fwd",
+            "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded ERA5-shaped smooth fields, random-init weights)",
+            "config": _describe(wl, K),
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": base["cores"],
+                             "kind": "oracle", "sample": base["sample"]},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

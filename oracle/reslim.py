@@ -17,11 +17,11 @@ What it computes (arxiv 2607.02829):
   (top-K by per-token L2 norm of the last dense-early block's output)
 * gather h0 = x[:, I, :] and the sparse middle blocks on h      -- Sec. 3.2 Eq. 8
 * the residual delta and scatter x' = x0 + Scatter(h - h0, I)   -- Sec. 3.2 Eq. 9
-* the pre-LN block h <- h + Attn(LN h); h <- h + MLP(LN h)       -- Sec. 3.3 Eq. 10
+* the pre-LN block h <- h + Attn(LN h); h <- h + MLP(LN h)       -- Sec. 3.3 Eq. 11
   with LayerNorm (eps 1e-5, affine), multi-head softmax attention with
   scale 1/sqrt(head_dim) and no mask, exact-erf GELU, MLP ratio 4
   (App. A, Table "architecture specification")
-* r = 1 is the plain dense stack                                -- Sec. 3.5 last paragraph
+* r = 1 is the plain dense stack                                -- Sec. 3.4, paragraph "Architecture-agnostic design"
 
 Parity pins: every function here is pinned by the ``-m "not gpu"`` tests
 (published SplitMix64 outputs, the K values the paper prints, brute-force
@@ -165,7 +165,7 @@ def attention(qkv: np.ndarray, heads: int, pool: Optional[ThreadPoolExecutor] = 
 
 def block(x: np.ndarray, w: Dict[str, np.ndarray], heads: int, eps: float = 1e-5,
           pool: Optional[ThreadPoolExecutor] = None) -> np.ndarray:
-    """One pre-LN ViT block on x [B, T, D] (Sec. 3.3 Eq. 10):
+    """One pre-LN ViT block on x [B, T, D] (Sec. 3.3 Eq. 11):
     x <- x + (Attn(LN1 x) Wo^T + bo);  x <- x + (GELU(LN2 x W1^T + b1) W2^T + b2)."""
     B, T, D = x.shape
     a = layer_norm(x, w["ln1_g"], w["ln1_b"], eps)
@@ -200,7 +200,7 @@ def forward(x: np.ndarray, weights: Sequence[Dict[str, np.ndarray]], n1: int, n2
     """The routed encoder of Alg. 1 (dense early, sparse middle, dense late) in fp64.
 
     x: [B, L, D]; weights: N = n1 + n2 + n3 dicts of block weights.
-    keep_ratio == 1 runs the plain dense stack (Sec. 3.5: r = 1 reverts to the
+    keep_ratio == 1 runs the plain dense stack (Sec. 3.4, "Architecture-agnostic design": r = 1 reverts to the
     dense baseline) unless ``bypass_dense`` is False, in which case the routed
     formulation runs with K = L (used only to check that the two agree).
     ``idx`` overrides the selector (used to re-run with given indices).

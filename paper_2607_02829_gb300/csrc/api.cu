@@ -1,0 +1,430 @@
+// C ABI of the Sparse-Reslim encoder forward: validation, workspace carve-up and
+// the launch sequence of Alg. 1 (dense early -> select -> gather -> sparse
+// middle -> delta scatter -> dense late).  Everything here is host code; every
+// step of the computation runs in the kernels it launches.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/sparse_reslim.h"
+#include "kernels.h"
+
+namespace sr {
+cudaError_t launch_gemm_simt(DType dt, Epi epi, const void* A, const void* Bw, int M, int N,
+                             int K, const EpiArgs& ea, cudaStream_t s);
+cudaError_t launch_attention_simt(DType dt, const void* qkv, void* out, int B, int T, int heads,
+                                  cudaStream_t s);
+}  // namespace sr
+
+using sr::DType;
+using sr::Epi;
+
+namespace {
+
+thread_local std::string g_last_msg;
+
+sr_status fail(sr_status st, const char* what) {
+  g_last_msg = what;
+  return st;
+}
+
+sr_status cuda_fail(cudaError_t e, const char* where) {
+  g_last_msg = std::string(where) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")";
+  return SR_ERR_CUDA;
+}
+
+#define SR_CUDA(call, where)                         \
+  do {                                               \
+    cudaError_t e__ = (call);                        \
+    if (e__ != cudaSuccess) return cuda_fail(e__, where); \
+  } while (0)
+
+constexpr size_t kAlign = 256;
+size_t align_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int32_t keep_count(int32_t L, float r) {
+  if (L < 1 || !(r > 0.0f) || !(r <= 1.0f)) return -1;
+  return static_cast<int32_t>(std::floor(static_cast<double>(r) * static_cast<double>(L)));
+}
+
+size_t elem_size(int32_t dtype) { return dtype == SR_BF16 ? 2 : 4; }
+
+// Workspace layout for a config and a maximum routed count Kmax.
+struct Plan {
+  size_t ln, qkv, att, u, h, idx, score, total;
+};
+
+Plan make_plan(const sr_config& c, int32_t Kmax) {
+  const size_t es = elem_size(c.dtype);
+  const size_t rows = size_t(c.B) * c.L;
+  const size_t rrows = size_t(c.B) * (Kmax > 0 ? Kmax : 0);
+  Plan p{};
+  size_t off = 0;
+  p.ln = off;    off += align_up(rows * c.D * es);
+  p.qkv = off;   off += align_up(rows * 3 * c.D * es);
+  p.att = off;   off += align_up(rows * c.D * es);
+  p.u = off;     off += align_up(rows * size_t(c.mlp_hidden) * es);
+  p.h = off;     off += align_up(rrows * c.D * es);
+  p.idx = off;   off += align_up(size_t(c.B) * c.L * sizeof(int32_t));
+  p.score = off; off += align_up(rows * sizeof(float));
+  p.total = off;
+  return p;
+}
+
+sr_status validate_config(const sr_config* c) {
+  if (!c) return fail(SR_ERR_INVALID_ARG, "config is NULL");
+  if (c->B < 1 || c->L < 1) return fail(SR_ERR_INVALID_ARG, "B and L must be >= 1");
+  if (c->heads < 1 || c->D != 64 * c->heads)
+    return fail(SR_ERR_UNSUPPORTED, "D must equal 64 * heads (head_dim 64)");
+  if (c->mlp_hidden < 64 || c->mlp_hidden % 64 != 0)
+    return fail(SR_ERR_UNSUPPORTED, "mlp_hidden must be a positive multiple of 64");
+  if (c->n1 < 0 || c->n2 < 0 || c->n3 < 0 || c->n1 + c->n2 + c->n3 < 1)
+    return fail(SR_ERR_INVALID_ARG, "block split needs n1, n2, n3 >= 0 and n1 + n2 + n3 >= 1");
+  if (c->dtype != SR_F32 && c->dtype != SR_BF16) return fail(SR_ERR_INVALID_ARG, "bad dtype");
+  if (c->selector != SR_SEL_RANDOM && c->selector != SR_SEL_TOPK_L2)
+    return fail(SR_ERR_INVALID_ARG, "bad selector");
+  if (c->shared_indices != 0 && c->shared_indices != 1)
+    return fail(SR_ERR_INVALID_ARG, "shared_indices must be 0 or 1");
+  if (!(c->ln_eps > 0.0f) || !std::isfinite(c->ln_eps))
+    return fail(SR_ERR_INVALID_ARG, "ln_eps must be a positive finite number");
+  const int maxD = c->dtype == SR_BF16 ? 2048 : 1024;
+  if (c->D > maxD) return fail(SR_ERR_UNSUPPORTED, "D too large for the row kernels");
+  if (c->L > sr::select_max_L())
+    return fail(SR_ERR_UNSUPPORTED, "L exceeds the selection kernel's shared-memory capacity");
+  const double rows = double(c->B) * double(c->L);
+  if (rows * double(c->mlp_hidden > 3 * c->D ? c->mlp_hidden : 3 * c->D) >= 2147483647.0)
+    return fail(SR_ERR_UNSUPPORTED, "B * L * width exceeds 2^31 elements");
+  return SR_OK;
+}
+
+}  // namespace
+
+struct TraceRec {
+  int kind;
+  cudaEvent_t ev0, ev1;
+  double flops, bytes;
+};
+
+struct sr_handle {
+  sr_config cfg;
+  DType dt;
+  size_t es;
+  char* ws;
+  size_t ws_bytes;
+  int32_t Kmax;
+  Plan plan;
+  bool trace = false;
+  std::vector<TraceRec> pending;
+  std::vector<cudaEvent_t> pool;
+  sr_trace_entry acc[SR_KERN_COUNT] = {};
+  void* at(size_t off) const { return ws + off; }
+  ~sr_handle() {
+    for (auto& r : pending) { cudaEventDestroy(r.ev0); cudaEventDestroy(r.ev1); }
+    for (auto e : pool) cudaEventDestroy(e);
+  }
+};
+
+namespace {
+
+cudaEvent_t take_event(sr_handle* h) {
+  if (!h->pool.empty()) {
+    cudaEvent_t e = h->pool.back();
+    h->pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+// Records CUDA events around one launch when the handle traces and the stream
+// is not capturing.
+struct TraceScope {
+  sr_handle* h;
+  cudaStream_t s;
+  TraceRec rec{};
+  bool on = false;
+  TraceScope(const sr_handle* hc, int kind, double flops, double bytes, cudaStream_t st)
+      : h(const_cast<sr_handle*>(hc)), s(st) {
+    if (!h->trace) return;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(s, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return;
+    rec.kind = kind; rec.flops = flops; rec.bytes = bytes;
+    rec.ev0 = take_event(h); rec.ev1 = take_event(h);
+    if (!rec.ev0 || !rec.ev1) return;
+    on = cudaEventRecord(rec.ev0, s) == cudaSuccess;
+  }
+  ~TraceScope() {
+    if (on && cudaEventRecord(rec.ev1, s) == cudaSuccess) h->pending.push_back(rec);
+  }
+};
+
+// GEMM and attention dispatch by dtype.
+cudaError_t gemm(const sr_handle* h, Epi epi, const void* A, const void* W, int M, int N, int K,
+                 const sr::EpiArgs& ea, cudaStream_t s) {
+  return sr::launch_gemm_simt(h->dt, epi, A, W, M, N, K, ea, s);
+}
+
+cudaError_t attention(const sr_handle* h, const void* qkv, void* out, int B, int T,
+                      cudaStream_t s) {
+  return sr::launch_attention_simt(h->dt, qkv, out, B, T, h->cfg.heads, s);
+}
+
+// One pre-LN block (Sec. 3.3 Eq. 11) on the residual stream x [B*T, D], in place.
+// With `scatter` set this is the last sparse block: its FC2 epilogue writes
+// x0 + (h_out - h0) into the rows idx of `scatter_out` [B*Lx, D] instead of x.
+sr_status run_block(const sr_handle* hd, void* x, int B, int T, const sr_block_weights& w,
+                    bool scatter, void* scatter_out, const int32_t* idx, int Lx,
+                    cudaStream_t s) {
+  const sr_config& c = hd->cfg;
+  const int rows = B * T, D = c.D, H = c.mlp_hidden;
+  const double es = double(hd->es), R = double(rows);
+  void* ln = hd->at(hd->plan.ln);
+  void* qkv = hd->at(hd->plan.qkv);
+  void* att = hd->at(hd->plan.att);
+  void* u = hd->at(hd->plan.u);
+  const double ln_bytes = (2.0 * R * D + 2.0 * D) * es;
+  {
+    TraceScope t(hd, SR_KERN_LAYERNORM, 0.0, ln_bytes, s);
+    SR_CUDA(sr::launch_layernorm(hd->dt, x, w.ln1_g, w.ln1_b, ln, rows, D, c.ln_eps, s), "layernorm1");
+  }
+  {
+    TraceScope t(hd, SR_KERN_GEMM_QKV, 2.0 * R * 3 * D * D,
+                 (R * D + 3.0 * D * D + R * 3 * D + 3.0 * D) * es, s);
+    sr::EpiArgs e1{w.bqkv, nullptr, qkv, nullptr, 0, 0};
+    SR_CUDA(gemm(hd, Epi::Bias, ln, w.wqkv, rows, 3 * D, D, e1, s), "qkv gemm");
+  }
+  {
+    TraceScope t(hd, SR_KERN_ATTENTION, 4.0 * B * c.heads * double(T) * T * 64.0,
+                 (R * 3 * D + R * D) * es, s);
+    SR_CUDA(attention(hd, qkv, att, B, T, s), "attention");
+  }
+  {
+    TraceScope t(hd, SR_KERN_GEMM_OUT, 2.0 * R * D * D, (R * D + 1.0 * D * D + 2.0 * R * D + D) * es, s);
+    sr::EpiArgs e2{w.bo, x, x, nullptr, 0, 0};
+    SR_CUDA(gemm(hd, Epi::BiasResidual, att, w.wo, rows, D, D, e2, s), "out-proj gemm");
+  }
+  {
+    TraceScope t(hd, SR_KERN_LAYERNORM, 0.0, ln_bytes, s);
+    SR_CUDA(sr::launch_layernorm(hd->dt, x, w.ln2_g, w.ln2_b, ln, rows, D, c.ln_eps, s), "layernorm2");
+  }
+  {
+    TraceScope t(hd, SR_KERN_GEMM_FC1, 2.0 * R * H * D, (R * D + 1.0 * H * D + R * H + H) * es, s);
+    sr::EpiArgs e3{w.b1, nullptr, u, nullptr, 0, 0};
+    SR_CUDA(gemm(hd, Epi::BiasGelu, ln, w.w1, rows, H, D, e3, s), "fc1 gemm");
+  }
+  if (!scatter) {
+    TraceScope t(hd, SR_KERN_GEMM_FC2, 2.0 * R * D * H, (R * H + 1.0 * D * H + 2.0 * R * D + D) * es, s);
+    sr::EpiArgs e4{w.b2, x, x, nullptr, 0, 0};
+    SR_CUDA(gemm(hd, Epi::BiasResidual, u, w.w2, rows, D, H, e4, s), "fc2 gemm");
+  } else {
+    // reads h and x0 rows, writes the scattered rows, plus the index set
+    TraceScope t(hd, SR_KERN_GEMM_FC2_SCATTER, 2.0 * R * D * H,
+                 (R * H + 1.0 * D * H + 3.0 * R * D + D) * es + 4.0 * R, s);
+    sr::EpiArgs e4{w.b2, x, scatter_out, idx, T, Lx};
+    SR_CUDA(gemm(hd, Epi::BiasResidualScatter, u, w.w2, rows, D, H, e4, s), "fc2 scatter gemm");
+  }
+  return SR_OK;
+}
+
+bool weights_ok(const sr_block_weights& w) {
+  const void* p[12] = {w.ln1_g, w.ln1_b, w.wqkv, w.bqkv, w.wo, w.bo,
+                       w.ln2_g, w.ln2_b, w.w1, w.b1, w.w2, w.b2};
+  for (const void* q : p)
+    if (!q || !aligned(q, 16)) return false;
+  return true;
+}
+
+sr_status do_select(sr_handle* h, const void* x, int32_t K, uint64_t seed, int32_t* idx,
+                    cudaStream_t s) {
+  const sr_config& c = h->cfg;
+  const double sel_bytes = 4.0 * c.B * K +
+      (c.selector == SR_SEL_TOPK_L2 ? double(c.B) * c.L * c.D * h->es : 0.0);
+  TraceScope t(h, SR_KERN_SELECT, 0.0, sel_bytes, s);
+  if (c.selector == SR_SEL_RANDOM) {
+    SR_CUDA(sr::launch_select_random(c.B, c.L, K, seed, c.shared_indices, idx, s), "select_random");
+  } else {
+    float* score = static_cast<float*>(h->at(h->plan.score));
+    SR_CUDA(sr::launch_token_sq_norms(h->dt, x, c.B * c.L, c.D, score, s), "token norms");
+    SR_CUDA(sr::launch_select_topk(c.B, c.L, K, score, idx, s), "select_topk");
+  }
+  return SR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t sr_keep_count(int32_t L, float keep_ratio) { return keep_count(L, keep_ratio); }
+
+size_t sr_workspace_bytes(const sr_config* cfg, float max_keep_ratio) {
+  if (validate_config(cfg) != SR_OK) return 0;
+  const int32_t K = keep_count(cfg->L, max_keep_ratio);
+  if (K < 0) return 0;
+  return make_plan(*cfg, K).total;
+}
+
+sr_status sr_create(const sr_config* cfg, void* workspace, size_t ws_bytes, sr_handle** out) {
+  if (!out) return fail(SR_ERR_INVALID_ARG, "out handle pointer is NULL");
+  *out = nullptr;
+  sr_status st = validate_config(cfg);
+  if (st != SR_OK) return st;
+  if (!workspace || !aligned(workspace, kAlign))
+    return fail(SR_ERR_WORKSPACE, "workspace is NULL or not 256-byte aligned");
+  // the largest Kmax whose plan fits: the routed buffers scale with Kmax
+  const Plan full = make_plan(*cfg, cfg->L);
+  int32_t Kmax = cfg->L;
+  if (ws_bytes < full.total) {
+    const Plan none = make_plan(*cfg, 0);
+    if (ws_bytes < none.total) return fail(SR_ERR_WORKSPACE, "workspace too small");
+    const size_t per_row = size_t(cfg->B) * cfg->D * elem_size(cfg->dtype);
+    Kmax = int32_t((ws_bytes - none.total) / (per_row ? per_row : 1));
+    while (Kmax > 0 && make_plan(*cfg, Kmax).total > ws_bytes) --Kmax;
+    if (Kmax < 1) return fail(SR_ERR_WORKSPACE, "workspace too small for any routed token");
+  }
+  sr_handle* h = new (std::nothrow) sr_handle;
+  if (!h) return fail(SR_ERR_INTERNAL, "host allocation failed");
+  h->cfg = *cfg;
+  h->dt = cfg->dtype == SR_BF16 ? DType::BF16 : DType::F32;
+  h->es = elem_size(cfg->dtype);
+  h->ws = static_cast<char*>(workspace);
+  h->ws_bytes = ws_bytes;
+  h->Kmax = Kmax;
+  h->plan = make_plan(*cfg, Kmax);
+  *out = h;
+  return SR_OK;
+}
+
+sr_status sr_destroy(sr_handle* h) {
+  delete h;
+  return SR_OK;
+}
+
+sr_status sr_select(sr_handle* h, const void* x, float keep_ratio, uint64_t seed, int32_t* idx,
+                    int32_t* K_out, void* stream) {
+  if (!h) return fail(SR_ERR_INVALID_ARG, "handle is NULL");
+  const int32_t K = keep_count(h->cfg.L, keep_ratio);
+  if (K < 0) return fail(SR_ERR_INVALID_ARG, "keep_ratio must lie in (0, 1]");
+  if (K < 1) return fail(SR_ERR_INVALID_ARG, "K = floor(L * keep_ratio) is 0");
+  if (!idx || !aligned(idx, 4)) return fail(SR_ERR_INVALID_ARG, "idx is NULL or misaligned");
+  if (h->cfg.selector == SR_SEL_TOPK_L2 && (!x || !aligned(x, 16)))
+    return fail(SR_ERR_INVALID_ARG, "top-K selection needs a 16-byte aligned x");
+  if (K_out) *K_out = K;
+  return do_select(h, x, K, seed, idx, static_cast<cudaStream_t>(stream));
+}
+
+sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, float keep_ratio,
+                     uint64_t seed, void* out, int32_t* idx_out, void* stream) {
+  if (!h) return fail(SR_ERR_INVALID_ARG, "handle is NULL");
+  const sr_config& c = h->cfg;
+  const int N = c.n1 + c.n2 + c.n3;
+  if (!x || !out || !aligned(x, 16) || !aligned(out, 16))
+    return fail(SR_ERR_INVALID_ARG, "x and out must be non-NULL and 16-byte aligned");
+  if (!w) return fail(SR_ERR_INVALID_ARG, "weights array is NULL");
+  for (int i = 0; i < N; ++i)
+    if (!weights_ok(w[i])) return fail(SR_ERR_INVALID_ARG, "a block weight pointer is NULL or misaligned");
+  if (idx_out && !aligned(idx_out, 4)) return fail(SR_ERR_INVALID_ARG, "idx_out misaligned");
+  const int32_t K = keep_count(c.L, keep_ratio);
+  if (K < 0) return fail(SR_ERR_INVALID_ARG, "keep_ratio must lie in (0, 1]");
+  const bool route = keep_ratio < 1.0f && c.n2 > 0;
+  if (K < 1 && (route || idx_out)) return fail(SR_ERR_INVALID_ARG, "K = floor(L * keep_ratio) is 0");
+  if (route && K > h->Kmax) return fail(SR_ERR_WORKSPACE, "K exceeds the workspace's routed capacity");
+  const size_t bytes = size_t(c.B) * c.L * c.D * h->es;
+  const char* xb = static_cast<const char*>(x);
+  char* ob = static_cast<char*>(out);
+  if (xb != ob && xb < ob + bytes && ob < xb + bytes)
+    return fail(SR_ERR_INVALID_ARG, "out partially overlaps x");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (xb != ob) {
+    TraceScope t(h, SR_KERN_COPY, 0.0, 2.0 * bytes, s);
+    SR_CUDA(cudaMemcpyAsync(out, x, bytes, cudaMemcpyDeviceToDevice, s), "copy x -> out");
+  }
+  sr_status st;
+  // stage 1: dense early
+  for (int i = 0; i < c.n1; ++i)
+    if ((st = run_block(h, out, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
+  int32_t* idx = idx_out ? idx_out : static_cast<int32_t*>(h->at(h->plan.idx));
+  if (route || idx_out)
+    if ((st = do_select(h, out, K, seed, idx, s)) != SR_OK) return st;
+  if (route) {
+    // stage 2: gather, sparse middle, delta scatter in the last block's epilogue
+    void* hbuf = h->at(h->plan.h);
+    {
+      TraceScope t(h, SR_KERN_GATHER, 0.0, 2.0 * c.B * K * c.D * h->es + 4.0 * c.B * K, s);
+      SR_CUDA(sr::launch_gather_rows(h->dt, out, idx, c.B, c.L, K, c.D, hbuf, s), "gather");
+    }
+    for (int i = c.n1; i < c.n1 + c.n2; ++i) {
+      const bool last = i == c.n1 + c.n2 - 1;
+      if ((st = run_block(h, hbuf, c.B, K, w[i], last, out, idx, c.L, s)) != SR_OK) return st;
+    }
+  } else {
+    for (int i = c.n1; i < c.n1 + c.n2; ++i)
+      if ((st = run_block(h, out, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
+  }
+  // stage 3: dense late
+  for (int i = c.n1 + c.n2; i < N; ++i)
+    if ((st = run_block(h, out, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
+  return SR_OK;
+}
+
+sr_status sr_forward_host(sr_handle* h, const void* x_host, const sr_block_weights* w,
+                          float keep_ratio, uint64_t seed, void* dev_xout, void* out_host,
+                          int32_t* idx_out, void* stream) {
+  if (!h) return fail(SR_ERR_INVALID_ARG, "handle is NULL");
+  if (!x_host || !out_host || !dev_xout)
+    return fail(SR_ERR_INVALID_ARG, "x_host, dev_xout and out_host must be non-NULL");
+  const sr_config& c = h->cfg;
+  const size_t bytes = size_t(c.B) * c.L * c.D * h->es;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  SR_CUDA(cudaMemcpyAsync(dev_xout, x_host, bytes, cudaMemcpyHostToDevice, s), "copy x host -> device");
+  sr_status st = sr_forward(h, dev_xout, w, keep_ratio, seed, dev_xout, idx_out, stream);
+  if (st != SR_OK) return st;
+  SR_CUDA(cudaMemcpyAsync(out_host, dev_xout, bytes, cudaMemcpyDeviceToHost, s), "copy out device -> host");
+  return SR_OK;
+}
+
+sr_status sr_trace_enable(sr_handle* h, int enable) {
+  if (!h) return fail(SR_ERR_INVALID_ARG, "handle is NULL");
+  h->trace = enable != 0;
+  return SR_OK;
+}
+
+sr_status sr_trace_read(sr_handle* h, sr_trace_entry* out, int reset) {
+  if (!h) return fail(SR_ERR_INVALID_ARG, "handle is NULL");
+  for (auto& r : h->pending) {
+    SR_CUDA(cudaEventSynchronize(r.ev1), "trace event sync");
+    float ms = 0.f;
+    SR_CUDA(cudaEventElapsedTime(&ms, r.ev0, r.ev1), "trace elapsed time");
+    sr_trace_entry& a = h->acc[r.kind];
+    a.ms += ms; a.launches += 1; a.flops += r.flops; a.bytes += r.bytes;
+    h->pool.push_back(r.ev0);
+    h->pool.push_back(r.ev1);
+  }
+  h->pending.clear();
+  if (out)
+    for (int k = 0; k < SR_KERN_COUNT; ++k) out[k] = h->acc[k];
+  if (reset)
+    for (int k = 0; k < SR_KERN_COUNT; ++k) h->acc[k] = sr_trace_entry{};
+  return SR_OK;
+}
+
+const char* sr_status_string(sr_status s) {
+  switch (s) {
+    case SR_OK: return "SR_OK";
+    case SR_ERR_INVALID_ARG: return "SR_ERR_INVALID_ARG: invalid argument";
+    case SR_ERR_UNSUPPORTED: return "SR_ERR_UNSUPPORTED: configuration not supported";
+    case SR_ERR_WORKSPACE: return "SR_ERR_WORKSPACE: workspace missing or too small";
+    case SR_ERR_CUDA: return "SR_ERR_CUDA: CUDA call failed";
+    case SR_ERR_INTERNAL: return "SR_ERR_INTERNAL: internal error";
+  }
+  return "unknown sr_status";
+}
+
+const char* sr_last_error_message(void) { return g_last_msg.c_str(); }
+
+}  // extern "C"

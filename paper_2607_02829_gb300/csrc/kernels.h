@@ -1,0 +1,59 @@
+// Internal launchers of the Sparse-Reslim CUDA library.  Every launcher only
+// enqueues work on `stream` and returns the launch's cudaError_t.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace sr {
+
+enum class DType : int { F32 = 0, BF16 = 1 };
+
+// ---- token selection (Sec. 3.2; App. B.2) --------------------------------
+// Random: K smallest SplitMix64 keys per sample (ties by index), sorted indices.
+cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared,
+                                 int32_t* idx, cudaStream_t s);
+// Squared L2 norm of every token of x [B*L, D] into score [B*L] (fp32).
+cudaError_t launch_token_sq_norms(DType dt, const void* x, int rows, int D, float* score,
+                                  cudaStream_t s);
+// K largest scores per sample (ties to the lower index), sorted indices.
+cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t* idx,
+                               cudaStream_t s);
+// Largest L the one-CTA-per-sample selection kernels accept (keys in shared memory).
+int select_max_L();
+
+// ---- gather (Eq. 8): h[b*K + k, :] = x[b*L + idx[b*K + k], :] ------------
+cudaError_t launch_gather_rows(DType dt, const void* x, const int32_t* idx, int B, int L, int K,
+                               int D, void* h, cudaStream_t s);
+
+// ---- LayerNorm over D: y = (x - mean) / sqrt(var + eps) * g + b -----------
+cudaError_t launch_layernorm(DType dt, const void* x, const void* g, const void* b, void* y,
+                             int rows, int D, float eps, cudaStream_t s);
+
+// ---- GEMM C = A B^T with fused epilogues ---------------------------------
+// A [M, K] row-major, B [N, K] row-major (nn.Linear weight), fp32 accumulate.
+enum class Epi : int {
+  Bias = 0,          // out[m, n] = acc + bias[n]
+  BiasGelu = 1,      // out[m, n] = GELU(acc + bias[n])
+  BiasResidual = 2,  // out[m, n] = res[m, n] + acc + bias[n]        (out may == res)
+  BiasResidualScatter = 3,  // hn = res[m, n] + acc + bias[n]; row m = b*Kr + k maps to
+                            // xrow = b*Lx + idx[m]; out[xrow, n] = x0 + (hn - x0), x0 = out[xrow, n]
+};
+struct EpiArgs {
+  const void* bias;     // [N]
+  const void* res;      // [M, N] (BiasResidual*)
+  void* out;            // [M, N], or [B*Lx, N] for the scatter epilogue
+  const int32_t* idx;   // [M] for the scatter epilogue
+  int Kr;               // routed rows per sample (scatter)
+  int Lx;               // tokens per sample of the scatter target
+};
+cudaError_t launch_gemm(DType dt, Epi epi, const void* A, const void* Bw, int M, int N, int K,
+                        const EpiArgs& ea, cudaStream_t s);
+
+// ---- attention core: per (sample, head) softmax(q k^T / sqrt(64)) v ------
+// qkv [B*T, 3D] (q | k | v, head h at columns 64h..64h+63 of each); out [B*T, D].
+cudaError_t launch_attention(DType dt, const void* qkv, void* out, int B, int T, int heads,
+                             cudaStream_t s);
+
+}  // namespace sr

@@ -1,0 +1,144 @@
+// Row-wise HBM-bound kernels: the routed-token gather (Eq. 8) and LayerNorm
+// (the LN of the pre-LN block, Sec. 3.3 Eq. 11).  One warp owns one row; rows
+// move as 16-byte vectors, all loads of a row are issued before any use.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace sr {
+namespace {
+
+// h[b*K + k, :] = x[b*L + idx[b*K + k], :]  -- a bit copy of D * sizeof(T) bytes.
+template <typename T, int NV>
+__global__ void __launch_bounds__(256)
+gather_rows_kernel(const T* __restrict__ x, const int32_t* __restrict__ idx, int L, int K,
+                   int D, int rows, T* __restrict__ h) {
+  constexpr int V = Elem<T>::kVec;
+  const int lane = threadIdx.x & 31;
+  const int nv = D / V;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += warps) {
+    const int b = r / K;
+    const int src = b * L + __ldg(idx + r);
+    const uint4* s = reinterpret_cast<const uint4*>(x + size_t(src) * D);
+    uint4* d = reinterpret_cast<uint4*>(h + size_t(r) * D);
+    uint4 v[NV];
+#pragma unroll
+    for (int j = 0; j < NV; ++j)
+      if (lane + 32 * j < nv) v[j] = __ldg(s + lane + 32 * j);
+#pragma unroll
+    for (int j = 0; j < NV; ++j)
+      if (lane + 32 * j < nv) d[lane + 32 * j] = v[j];
+  }
+}
+
+// y = (x - mean) / sqrt(var + eps) * g + b, statistics in fp32, two passes over
+// the row held in registers (biased variance).
+template <typename T, int NV>
+__global__ void __launch_bounds__(256)
+layernorm_kernel(const T* __restrict__ x, const T* __restrict__ g, const T* __restrict__ bta,
+                 T* __restrict__ y, int rows, int D, float eps) {
+  constexpr int V = Elem<T>::kVec;
+  const int lane = threadIdx.x & 31;
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  if (row >= rows) return;
+  const int nv = D / V;
+  const uint4* xr = reinterpret_cast<const uint4*>(x + size_t(row) * D);
+  float f[NV][V];
+  float sum = 0.f;
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    if (lane + 32 * j < nv) {
+      unpack16(__ldg(xr + lane + 32 * j), f[j]);
+#pragma unroll
+      for (int e = 0; e < V; ++e) sum += f[j][e];
+    }
+  }
+  const float mean = warp_sum(sum) / float(D);
+  float sq = 0.f;
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    if (lane + 32 * j < nv) {
+#pragma unroll
+      for (int e = 0; e < V; ++e) { const float c = f[j][e] - mean; sq = fmaf(c, c, sq); }
+    }
+  }
+  const float rstd = rsqrtf(warp_sum(sq) / float(D) + eps);
+  const uint4* gr = reinterpret_cast<const uint4*>(g);
+  const uint4* br = reinterpret_cast<const uint4*>(bta);
+  uint4* yr = reinterpret_cast<uint4*>(y + size_t(row) * D);
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    const int v = lane + 32 * j;
+    if (v < nv) {
+      float gf[V], bf[V], o[V];
+      unpack16(__ldg(gr + v), gf);
+      unpack16(__ldg(br + v), bf);
+#pragma unroll
+      for (int e = 0; e < V; ++e) o[e] = (f[j][e] - mean) * rstd * gf[e] + bf[e];
+      yr[v] = pack16(o);
+    }
+  }
+}
+
+template <typename T, int NV>
+cudaError_t gather_t(const void* x, const int32_t* idx, int B, int L, int K, int D, void* h,
+                     cudaStream_t s) {
+  const int rows = B * K;
+  int blocks = (rows + 7) / 8;
+  if (blocks > 152 * 16) blocks = 152 * 16;
+  gather_rows_kernel<T, NV><<<blocks, 256, 0, s>>>(static_cast<const T*>(x), idx, L, K, D, rows,
+                                                   static_cast<T*>(h));
+  return cudaGetLastError();
+}
+
+template <typename T, int NV>
+cudaError_t layernorm_t(const void* x, const void* g, const void* b, void* y, int rows, int D,
+                        float eps, cudaStream_t s) {
+  layernorm_kernel<T, NV><<<(rows + 7) / 8, 256, 0, s>>>(
+      static_cast<const T*>(x), static_cast<const T*>(g), static_cast<const T*>(b),
+      static_cast<T*>(y), rows, D, eps);
+  return cudaGetLastError();
+}
+
+// vectors per lane needed for a row of D elements
+template <typename T> int lanes_nv(int D) { return (D / Elem<T>::kVec + 31) / 32; }
+
+}  // namespace
+
+cudaError_t launch_gather_rows(DType dt, const void* x, const int32_t* idx, int B, int L, int K,
+                               int D, void* h, cudaStream_t s) {
+  if (dt == DType::BF16) {
+    const int nv = lanes_nv<bf16>(D);
+    if (nv <= 1) return gather_t<bf16, 1>(x, idx, B, L, K, D, h, s);
+    if (nv <= 2) return gather_t<bf16, 2>(x, idx, B, L, K, D, h, s);
+    if (nv <= 4) return gather_t<bf16, 4>(x, idx, B, L, K, D, h, s);
+    if (nv <= 8) return gather_t<bf16, 8>(x, idx, B, L, K, D, h, s);
+  } else {
+    const int nv = lanes_nv<float>(D);
+    if (nv <= 1) return gather_t<float, 1>(x, idx, B, L, K, D, h, s);
+    if (nv <= 2) return gather_t<float, 2>(x, idx, B, L, K, D, h, s);
+    if (nv <= 4) return gather_t<float, 4>(x, idx, B, L, K, D, h, s);
+    if (nv <= 8) return gather_t<float, 8>(x, idx, B, L, K, D, h, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_layernorm(DType dt, const void* x, const void* g, const void* b, void* y,
+                             int rows, int D, float eps, cudaStream_t s) {
+  if (dt == DType::BF16) {
+    const int nv = lanes_nv<bf16>(D);
+    if (nv <= 1) return layernorm_t<bf16, 1>(x, g, b, y, rows, D, eps, s);
+    if (nv <= 2) return layernorm_t<bf16, 2>(x, g, b, y, rows, D, eps, s);
+    if (nv <= 4) return layernorm_t<bf16, 4>(x, g, b, y, rows, D, eps, s);
+    if (nv <= 8) return layernorm_t<bf16, 8>(x, g, b, y, rows, D, eps, s);
+  } else {
+    const int nv = lanes_nv<float>(D);
+    if (nv <= 1) return layernorm_t<float, 1>(x, g, b, y, rows, D, eps, s);
+    if (nv <= 2) return layernorm_t<float, 2>(x, g, b, y, rows, D, eps, s);
+    if (nv <= 4) return layernorm_t<float, 4>(x, g, b, y, rows, D, eps, s);
+    if (nv <= 8) return layernorm_t<float, 8>(x, g, b, y, rows, D, eps, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace sr

@@ -1,0 +1,211 @@
+// Token selection (Sec. 3.2 random selection; App. B.2 activation-norm selector).
+//
+// Both selectors reduce to one primitive: per sample, keep the K smallest keys
+// (ties broken by the lower token index) and emit their token indices in
+// ascending order.  One CTA owns one sample: its L keys sit in shared memory, a
+// most-significant-digit radix select (8-bit digits) finds the K-th smallest key
+// T and how many keys equal to T must be kept, and an ordered block-wide
+// compaction writes the selected indices, which come out sorted by
+// construction.  Work per sample is O(L * passes); HBM traffic is the index
+// write (4 B per selected token) plus, for the top-K selector, one read of x.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace sr {
+namespace {
+
+constexpr int kSelThreads = 1024;
+constexpr int kSelMaxL = 24576;   // 192 KB of 8-byte keys in shared memory
+
+// SplitMix64 output function (Steele, Lea & Flood, OOPSLA 2014).
+__device__ __forceinline__ uint64_t splitmix64_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Scores in descending order become keys in ascending order (equal scores give
+// equal keys, so ties fall to the index order of the compaction).
+__device__ __forceinline__ uint32_t desc_key(float score) {
+  uint32_t u = __float_as_uint(score);
+  uint32_t asc = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  return ~asc;
+}
+
+// Block-wide exclusive prefix count of `flag` in thread order; returns the
+// thread's exclusive prefix and writes the block total to *total.
+__device__ __forceinline__ int block_excl_count(bool flag, int* warp_tot, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const unsigned bal = __ballot_sync(0xffffffffu, flag);
+  const int in_warp = __popc(bal & ((1u << lane) - 1u));
+  if (lane == 0) warp_tot[warp] = __popc(bal);
+  __syncthreads();
+  if (warp == 0) {
+    const int nw = blockDim.x >> 5;
+    int v = lane < nw ? warp_tot[lane] : 0;
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (lane < nw) warp_tot[lane] = incl - v;   // exclusive warp offsets
+    if (lane == 31) *total = incl;
+  }
+  __syncthreads();
+  const int r = warp_tot[warp] + in_warp;
+  __syncthreads();   // warp_tot is reused by the next call
+  return r;
+}
+
+template <typename Key>
+__device__ void select_smallest_sorted(const Key* keys, int L, int K, int32_t* out_idx) {
+  __shared__ int hist[256];
+  __shared__ int warp_tot[32];
+  __shared__ int s_total;
+  __shared__ Key s_prefix;
+  __shared__ int s_krem;
+  const int tid = threadIdx.x;
+  if (tid == 0) { s_prefix = 0; s_krem = K; }
+  Key mask = 0;
+  __syncthreads();
+  // ---- radix select of the K-th smallest key, most significant digit first
+  for (int shift = int(sizeof(Key) * 8) - 8; shift >= 0; shift -= 8) {
+    for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    const Key prefix = s_prefix;
+    for (int i = tid; i < L; i += blockDim.x) {
+      const Key k = keys[i];
+      if ((k & mask) == prefix) atomicAdd(&hist[int((k >> shift) & 0xff)], 1);
+    }
+    __syncthreads();
+    if (tid < 32) {
+      // lane l owns bins 8l .. 8l+7
+      int c[8], s = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) { c[j] = hist[8 * tid + j]; s += c[j]; }
+      int incl = s;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        int t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (tid >= o) incl += t;
+      }
+      const int krem = s_krem;
+      const int excl = incl - s;
+      const bool mine = excl < krem && krem <= incl;
+      const unsigned who = __ballot_sync(0xffffffffu, mine);
+      if (mine) {
+        int acc = excl, d = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (acc + c[j] >= krem) { d = j; break; }
+          acc += c[j];
+        }
+        s_prefix = prefix | (Key(8 * tid + d) << shift);
+        s_krem = krem - acc;
+      }
+      (void)who;
+    }
+    mask |= Key(0xff) << shift;
+    __syncthreads();
+  }
+  const Key T = s_prefix;      // the K-th smallest key
+  const int keep_eq = s_krem;  // how many keys equal to T are kept (lowest indices first)
+  // ---- ordered compaction: keep key < T, and the first keep_eq keys == T
+  int eq_base = 0, out_base = 0;
+  for (int base = 0; base < L; base += blockDim.x) {
+    const int i = base + tid;
+    const Key k = i < L ? keys[i] : Key(0);
+    const bool is_eq = i < L && k == T;
+    const int eq_rank = eq_base + block_excl_count(is_eq, warp_tot, &s_total);
+    const int eq_tot = s_total;
+    const bool keep = i < L && (k < T || (is_eq && eq_rank < keep_eq));
+    const int pos = out_base + block_excl_count(keep, warp_tot, &s_total);
+    const int keep_tot = s_total;
+    if (keep) out_idx[pos] = i;
+    eq_base += eq_tot;
+    out_base += keep_tot;
+    __syncthreads();
+  }
+}
+
+__global__ void __launch_bounds__(kSelThreads)
+select_random_kernel(int L, int K, uint64_t seed, int shared, int32_t* idx) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  uint64_t* keys = reinterpret_cast<uint64_t*>(smem_raw);
+  const int b = blockIdx.x;
+  const uint64_t bb = shared ? 0ull : uint64_t(b);
+  for (int i = threadIdx.x; i < L; i += blockDim.x) {
+    const uint64_t ctr = 1ull + bb * uint64_t(L) + uint64_t(i);
+    keys[i] = splitmix64_mix(seed + 0x9E3779B97F4A7C15ull * ctr);
+  }
+  __syncthreads();
+  select_smallest_sorted<uint64_t>(keys, L, K, idx + size_t(b) * K);
+}
+
+__global__ void __launch_bounds__(kSelThreads)
+select_topk_kernel(int L, int K, const float* __restrict__ score, int32_t* idx) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  uint32_t* keys = reinterpret_cast<uint32_t*>(smem_raw);
+  const int b = blockIdx.x;
+  for (int i = threadIdx.x; i < L; i += blockDim.x) keys[i] = desc_key(score[size_t(b) * L + i]);
+  __syncthreads();
+  select_smallest_sorted<uint32_t>(keys, L, K, idx + size_t(b) * K);
+}
+
+// One warp per token: fp32 sum of squares over D, 16-byte loads.
+template <typename T>
+__global__ void __launch_bounds__(256)
+token_sq_norms_kernel(const T* __restrict__ x, int rows, int D, float* __restrict__ score) {
+  constexpr int V = Elem<T>::kVec;
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= rows) return;
+  const uint4* row = reinterpret_cast<const uint4*>(x + size_t(warp) * D);
+  const int nv = D / V;
+  float acc = 0.f;
+  for (int v = lane; v < nv; v += 32) {
+    float f[V];
+    unpack16(__ldg(row + v), f);
+#pragma unroll
+    for (int j = 0; j < V; ++j) acc = fmaf(f[j], f[j], acc);
+  }
+  acc = warp_sum(acc);
+  if (lane == 0) score[warp] = acc;
+}
+
+}  // namespace
+
+int select_max_L() { return kSelMaxL; }
+
+cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared, int32_t* idx,
+                                 cudaStream_t s) {
+  const size_t smem = size_t(L) * sizeof(uint64_t);
+  cudaError_t e = cudaFuncSetAttribute(select_random_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  select_random_kernel<<<B, kSelThreads, smem, s>>>(L, K, seed, shared, idx);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t* idx,
+                               cudaStream_t s) {
+  const size_t smem = size_t(L) * sizeof(uint32_t);
+  cudaError_t e = cudaFuncSetAttribute(select_topk_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  select_topk_kernel<<<B, kSelThreads, smem, s>>>(L, K, score, idx);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_token_sq_norms(DType dt, const void* x, int rows, int D, float* score,
+                                  cudaStream_t s) {
+  const int blocks = (rows + 7) / 8;
+  if (dt == DType::BF16)
+    token_sq_norms_kernel<bf16><<<blocks, 256, 0, s>>>(static_cast<const bf16*>(x), rows, D, score);
+  else
+    token_sq_norms_kernel<float><<<blocks, 256, 0, s>>>(static_cast<const float*>(x), rows, D, score);
+  return cudaGetLastError();
+}
+
+}  // namespace sr

@@ -1,0 +1,107 @@
+"""Host-side checks of the C ABI that need no GPU: the library loads, exports
+every function include/*.h declares, and rejects invalid arguments before any
+CUDA call."""
+import ctypes
+
+import pytest
+
+from tests._helpers import built_lib, header_functions
+
+
+@pytest.fixture(scope="module")
+def L():
+    return built_lib()
+
+
+def test_exports_every_declared_function(L):
+    names = header_functions()
+    assert "sr_forward" in names and "sr_create" in names
+    for n in names:
+        assert hasattr(L, n), f"{n} declared in include/ but not exported"
+
+
+def test_keep_count(L):
+    from paper_2607_02829_gb300 import binding as b
+    assert b.sr_keep_count(16200, 0.25) == 4050
+    assert b.sr_keep_count(8192, 0.25) == 2048
+    assert b.sr_keep_count(2048, 0.125) == 256
+    assert b.sr_keep_count(10, 0.0) == -1
+    assert b.sr_keep_count(10, 1.5) == -1
+    assert b.sr_keep_count(10, float("nan")) == -1
+    assert b.sr_keep_count(0, 0.5) == -1
+    assert b.sr_keep_count(3, 0.3) == 0
+
+
+def test_invalid_configs_rejected(L):
+    from paper_2607_02829_gb300 import binding as b
+    good = b.make_config(2, 512, 256, 4, 2, 2, 2, dtype="f32")
+    assert b.sr_workspace_bytes(good, 0.25) > 0
+    bad = [
+        dict(D=250), dict(heads=3), dict(B=0), dict(L=0), dict(n1=-1),
+        dict(n1=0, n2=0, n3=0), dict(dtype=7), dict(selector=5), dict(shared_indices=2),
+        dict(ln_eps=0.0), dict(mlp_hidden=100), dict(L=100000),
+    ]
+    for kw in bad:
+        c = b.make_config(2, 512, 256, 4, 2, 2, 2, dtype="f32")
+        for k, v in kw.items():
+            setattr(c, k, v)
+        assert b.sr_workspace_bytes(c, 0.25) == 0, kw
+
+
+def _handle(b, cfg, nbytes):
+    # a fake, 256-byte aligned device address: sr_create only records it
+    return b.sr_create(cfg, 0x100000, nbytes)
+
+
+def test_create_and_argument_errors(L):
+    from paper_2607_02829_gb300 import binding as b
+    cfg = b.make_config(2, 512, 256, 4, 2, 2, 2, dtype="f32")
+    n = b.sr_workspace_bytes(cfg, 0.25)
+    with pytest.raises(b.SRError) as e:
+        b.sr_create(cfg, 0, n)
+    assert e.value.status == b.SR_ERR_WORKSPACE
+    with pytest.raises(b.SRError) as e:
+        b.sr_create(cfg, 0x100001, n)
+    assert e.value.status == b.SR_ERR_WORKSPACE
+    with pytest.raises(b.SRError) as e:
+        b.sr_create(cfg, 0x100000, 1000)
+    assert e.value.status == b.SR_ERR_WORKSPACE
+    h = _handle(b, cfg, n)
+    try:
+        w = (b.sr_block_weights * 6)()
+        for i in range(6):
+            for f in b.WEIGHT_FIELDS:
+                setattr(w[i], f, 0x200000)
+        X, O = 0x400000, 0x800000
+        for r in (0.0, -1.0, 1.5, float("nan")):
+            with pytest.raises(b.SRError) as e:
+                b.sr_forward(h, X, w, r, 0, O, None, None)
+            assert e.value.status == b.SR_ERR_INVALID_ARG
+        # K = floor(512 * 0.001) = 0
+        with pytest.raises(b.SRError) as e:
+            b.sr_forward(h, X, w, 0.001, 0, O, None, None)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+        # beyond the workspace's routed capacity (sized for r <= 0.25)
+        with pytest.raises(b.SRError) as e:
+            b.sr_forward(h, X, w, 0.5, 0, O, None, None)
+        assert e.value.status == b.SR_ERR_WORKSPACE
+        # partial overlap of x and out
+        with pytest.raises(b.SRError) as e:
+            b.sr_forward(h, X, w, 0.25, 0, X + 1024, None, None)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+        # a NULL weight pointer
+        w[3].w1 = None
+        with pytest.raises(b.SRError) as e:
+            b.sr_forward(h, X, w, 0.25, 0, O, None, None)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+        with pytest.raises(b.SRError) as e:
+            b.sr_select(h, None, 0.0, 0, 0x300000, None)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+    finally:
+        b.sr_destroy(h)
+
+
+def test_status_strings(L):
+    from paper_2607_02829_gb300 import binding as b
+    for s in range(6):
+        assert L.sr_status_string(s).decode().startswith("SR_")

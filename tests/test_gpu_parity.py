@@ -1,0 +1,173 @@
+"""GPU parity of the CUDA path (through the C ABI) against the fp64 oracle.
+
+Bars: indices and the unselected-token passthrough bit-exact; outputs within a
+max-norm relative error max|y - o| / max|o| of 1e-4 (fp32) or 2e-2 (bf16).
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import reslim as o
+from paper_2607_02829_gb300 import synth
+from tests._helpers import built_lib, gpu_forward, max_norm_rel
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"f32": 1e-4, "bf16": 2e-2}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.fail("CUDA GPU required for -m gpu tests")
+    built_lib()
+
+
+def _oracle(wl, x, ws, keep_ratio=None, seed=None, selector=None, n_split=None, idx=None):
+    n1, n2, n3 = n_split or (wl.n1, wl.n2, wl.n3)
+    xf = synth.stored_as_f64(x)
+    wf = o.as_f64_weights(ws[:n1 + n2 + n3])
+    return o.forward(xf, wf, n1, n2, n3, wl.heads,
+                     wl.keep_ratio if keep_ratio is None else keep_ratio,
+                     seed=wl.select_seed if seed is None else seed,
+                     selector=selector or wl.selector, idx=idx, threads=8)
+
+
+def _tiny(dtype, B=2, L=200, heads=2, split=(1, 2, 1), r=0.25, selector="random"):
+    return synth.Workload(f"tiny_{dtype}", B=B, grid_h=1, grid_w=L, channels=3, patch=1,
+                          D=64 * heads, heads=heads, n1=split[0], n2=split[1], n3=split[2],
+                          keep_ratio=r, dtype=dtype, selector=selector, seed_index=77)
+
+
+# ------------------------------------------------------------ selection
+@pytest.mark.parametrize("B,L,K,shared", [
+    (1, 1, 1, False), (3, 10, 4, False), (2, 512, 128, False), (32, 512, 128, False),
+    (8, 2048, 512, False), (8, 2048, 2048, False), (1, 16200, 4050, False),
+    (4, 1000, 1, True), (2, 24576, 6144, False), (5, 777, 776, True)])
+def test_select_random_bitexact(B, L, K, shared):
+    from paper_2607_02829_gb300 import binding as b
+    cfg = b.make_config(B, L, 64, 1, 0, 1, 0, dtype="bf16", shared=shared)
+    for seed in (0, 3004, 2**64 - 1):
+        enc = b.Encoder(cfg, max_keep_ratio=1.0)
+        r = K / L
+        assert b.sr_keep_count(L, r) == K
+        idx = enc.select(None, r, seed).cpu().numpy()
+        torch.cuda.synchronize()
+        expect = o.select_random(B, L, K, seed, shared)
+        assert np.array_equal(idx, expect)
+        enc.close()
+
+
+@pytest.mark.parametrize("B,L,D,K,dtype", [(2, 300, 64, 75, "bf16"), (8, 2048, 1024, 512, "bf16"),
+                                           (1, 16200, 1024, 4050, "bf16"), (2, 512, 256, 128, "f32")])
+def test_select_topk_l2(B, L, D, K, dtype):
+    from paper_2607_02829_gb300 import binding as b
+    g = torch.Generator().manual_seed(B * L + D)
+    x = torch.randn(B, L, D, generator=g, dtype=torch.float64)
+    x[:, 1::7] = x[:, 0::7][:, :x[:, 1::7].shape[1]]           # exact duplicate rows -> exact ties
+    xs = x.to(synth.torch_dtype(dtype))
+    cfg = b.make_config(B, L, D, D // 64, 0, 1, 0, dtype=dtype, selector="topk_l2")
+    enc = b.Encoder(cfg, max_keep_ratio=1.0)
+    idx = enc.select(xs.cuda(), K / L, 0).cpu().numpy()
+    enc.close()
+    xf = synth.stored_as_f64(xs)
+    expect = o.select_topk_l2(xf, K)
+    s = o.token_sq_norms(xf)
+    for bb in range(B):
+        assert np.all(np.diff(idx[bb]) > 0) and idx[bb].min() >= 0 and idx[bb].max() < L
+        got, exp = set(idx[bb].tolist()), set(expect[bb].tolist())
+        if got == exp:
+            continue
+        # the GPU ranks fp32 sums: a disagreement is only allowed inside the band of
+        # fp32 rounding around the K-th score
+        kth = np.sort(s[bb])[::-1][K - 1]
+        for i in got ^ exp:
+            assert abs(s[bb, i] - kth) <= 1e-5 * kth, (i, s[bb, i], kth)
+
+
+# ------------------------------------------------- routing invariants (GPU)
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_zero_sparse_blocks_give_exact_passthrough(dtype):
+    # sparse blocks with all W and b zero add exactly 0: h == h0, delta == 0,
+    # and x' == x0 everywhere -- checks gather and scatter addressing bit-exactly
+    wl = _tiny(dtype, split=(1, 2, 0))
+    x, ws = synth.make_inputs(wl)
+    for i in (1, 2):
+        ws[i] = {k: (v if k.endswith("_g") else torch.zeros_like(v)) for k, v in ws[i].items()}
+    out, idx = gpu_forward(wl, x, ws)
+    x0, _ = gpu_forward(wl, x, ws, n_split=(1, 0, 0), want_idx=False)
+    assert torch.equal(out, x0)
+    assert idx.shape == (wl.B, 50)
+
+
+@pytest.mark.parametrize("wlname", ["c1_5p625deg_f32", "c2_5p625deg_bf16"])
+def test_unselected_tokens_bitexact(wlname):
+    wl = synth.WORKLOADS[wlname]
+    x, ws = synth.make_inputs(wl)
+    out, idx = gpu_forward(wl, x, ws, n_split=(wl.n1, wl.n2, 0))
+    x0, _ = gpu_forward(wl, x, ws, n_split=(wl.n1, 0, 0), want_idx=False)
+    assert np.array_equal(idx, o.select_random(wl.B, wl.L, wl.L // 4, wl.select_seed))
+    sel = np.zeros((wl.B, wl.L), dtype=bool)
+    sel[np.arange(wl.B)[:, None], idx] = True
+    assert torch.equal(out[torch.from_numpy(~sel)], x0[torch.from_numpy(~sel)])
+    changed = (out != x0).any(dim=-1)
+    assert changed[torch.from_numpy(sel)].float().mean() > 0.99
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_r1_is_bitwise_the_dense_stack(dtype):
+    wl = _tiny(dtype, split=(1, 2, 1))
+    x, ws = synth.make_inputs(wl)
+    a, _ = gpu_forward(wl, x, ws, keep_ratio=1.0, want_idx=False)
+    d, _ = gpu_forward(wl, x, ws, keep_ratio=1.0, n_split=(4, 0, 0), want_idx=False)
+    assert torch.equal(a, d)
+
+
+def test_in_place_equals_out_of_place():
+    wl = _tiny("bf16")
+    x, ws = synth.make_inputs(wl)
+    a, ia = gpu_forward(wl, x, ws)
+    b_, ib = gpu_forward(wl, x, ws, inplace=True)
+    assert torch.equal(a, b_) and np.array_equal(ia, ib)
+
+
+# ------------------------------------------------------ end-to-end parity
+@pytest.mark.parametrize("dtype,B,L,heads,split,r", [
+    ("f32", 2, 200, 2, (1, 2, 1), 0.25),
+    ("bf16", 2, 200, 2, (1, 2, 1), 0.25),
+    ("bf16", 3, 333, 4, (1, 3, 1), 0.5),      # ragged tiles everywhere
+    ("bf16", 1, 1, 1, (1, 1, 1), 1.0),        # a single token
+    ("bf16", 2, 129, 2, (0, 2, 0), 0.125),    # K = 16, routing only
+    ("f32", 1, 97, 1, (2, 1, 0), 0.5),
+])
+def test_forward_parity_small(dtype, B, L, heads, split, r):
+    wl = _tiny(dtype, B=B, L=L, heads=heads, split=split, r=r)
+    x, ws = synth.make_inputs(wl)
+    out, idx = gpu_forward(wl, x, ws, want_idx=r < 1.0)
+    ref, ridx = _oracle(wl, x, ws)
+    if r < 1.0:
+        assert np.array_equal(idx, ridx)
+    err = max_norm_rel(synth.stored_as_f64(out), ref)
+    assert err <= TOL[dtype], err
+
+
+@pytest.mark.parametrize("wlname", ["c1_5p625deg_f32", "c2_5p625deg_bf16"])
+def test_forward_parity_workload(wlname):
+    wl = synth.WORKLOADS[wlname]
+    x, ws = synth.make_inputs(wl)
+    out, idx = gpu_forward(wl, x, ws)
+    ref, ridx = _oracle(wl, x, ws)
+    assert np.array_equal(idx, ridx)
+    err = max_norm_rel(synth.stored_as_f64(out), ref)
+    assert err <= TOL[wl.dtype], err
+
+
+def test_forward_parity_topk_selector_small():
+    wl = _tiny("bf16", B=2, L=256, heads=2, split=(1, 2, 1), r=0.25, selector="topk_l2")
+    x, ws = synth.make_inputs(wl)
+    out, idx = gpu_forward(wl, x, ws)
+    ref, ridx = _oracle(wl, x, ws, idx=idx)      # same indices on both sides
+    err = max_norm_rel(synth.stored_as_f64(out), ref)
+    assert err <= TOL["bf16"], err
+    x0, _ = gpu_forward(wl, x, ws, n_split=(1, 0, 0), want_idx=False)
+    assert np.array_equal(idx, o.select_topk_l2(synth.stored_as_f64(x0), 64))

@@ -202,7 +202,7 @@ def _torch_block(w, D, H, hidden):
 
 def test_block_against_torch_prenorm_encoder_layer():
     # PyTorch's TransformerEncoderLayer with norm_first=True is the pre-LN block
-    # of Eq. 10 (packed q/k/v in_proj, per-head column groups, 1/sqrt(dh) scale).
+    # of Eq. 11 (packed q/k/v in_proj, per-head column groups, 1/sqrt(dh) scale).
     rng = np.random.default_rng(5)
     B, T, D, H = 2, 11, 32, 4
     w = _rand_weights(rng, D, 4 * D)
