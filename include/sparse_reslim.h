@@ -178,6 +178,15 @@ sr_status sr_destroy(sr_handle* h);
 /* Static description of a status code. */
 const char* sr_status_string(sr_status s);
 
+/* Reads the handle's device fault word (kept in its workspace) into *fault
+ * (host) after the work enqueued on `stream` so far, resetting it when
+ * clear != 0.  Bit 0 set means a tensor-core kernel of that handle gave up
+ * waiting on one of its pipeline barriers (each wait is bounded to 2 s) and
+ * returned early, so the outputs of that call are invalid.  The handle's first
+ * sr_forward zeroes the word; afterwards it stays set until cleared here.
+ * Synchronises `stream`. */
+sr_status sr_device_fault(sr_handle* h, uint32_t* fault, int clear, void* stream);
+
 /* The last CUDA or validation message recorded on this thread ("" if none). */
 const char* sr_last_error_message(void);
 

@@ -79,6 +79,8 @@ def lib() -> ctypes.CDLL:
         L.sr_trace_enable.argtypes = [vp, ctypes.c_int]; L.sr_trace_enable.restype = st
         L.sr_trace_read.argtypes = [vp, ctypes.POINTER(sr_trace_entry), ctypes.c_int]
         L.sr_trace_read.restype = st
+        L.sr_device_fault.argtypes = [vp, ctypes.POINTER(ctypes.c_uint32), ctypes.c_int, vp]
+        L.sr_device_fault.restype = st
         L.sr_status_string.argtypes = [st]; L.sr_status_string.restype = ctypes.c_char_p
         L.sr_last_error_message.argtypes = []; L.sr_last_error_message.restype = ctypes.c_char_p
         _lib = L
@@ -141,6 +143,13 @@ def sr_trace_read(handle: int, reset: bool = True) -> dict:
     _check(lib().sr_trace_read(handle, arr, int(bool(reset))), "sr_trace_read")
     return {k: {"ms": e.ms, "launches": e.launches, "flops": e.flops, "bytes": e.bytes}
             for k, e in zip(KERNEL_KINDS, arr)}
+
+
+def sr_device_fault(handle: int, clear: bool, stream: int) -> int:
+    f = ctypes.c_uint32(0)
+    _check(lib().sr_device_fault(handle, ctypes.byref(f), int(bool(clear)), stream),
+           "sr_device_fault")
+    return f.value
 
 
 # ----------------------------------------------------- torch-side helpers

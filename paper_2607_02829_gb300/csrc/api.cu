@@ -12,13 +12,6 @@
 #include "../../include/sparse_reslim.h"
 #include "kernels.h"
 
-namespace sr {
-cudaError_t launch_gemm_simt(DType dt, Epi epi, const void* A, const void* Bw, int M, int N,
-                             int K, const EpiArgs& ea, cudaStream_t s);
-cudaError_t launch_attention_simt(DType dt, const void* qkv, void* out, int B, int T, int heads,
-                                  cudaStream_t s);
-}  // namespace sr
-
 using sr::DType;
 using sr::Epi;
 
@@ -56,7 +49,7 @@ size_t elem_size(int32_t dtype) { return dtype == SR_BF16 ? 2 : 4; }
 
 // Workspace layout for a config and a maximum routed count Kmax.
 struct Plan {
-  size_t ln, qkv, att, u, h, idx, score, total;
+  size_t fault, xs, ln, qkv, att, u, hs, idx, score, total;
 };
 
 Plan make_plan(const sr_config& c, int32_t Kmax) {
@@ -65,11 +58,13 @@ Plan make_plan(const sr_config& c, int32_t Kmax) {
   const size_t rrows = size_t(c.B) * (Kmax > 0 ? Kmax : 0);
   Plan p{};
   size_t off = 0;
+  p.fault = off; off += kAlign;                                   // device fault word
+  p.xs = off;    off += align_up(rows * c.D * sizeof(float));     // fp32 residual stream
   p.ln = off;    off += align_up(rows * c.D * es);
   p.qkv = off;   off += align_up(rows * 3 * c.D * es);
   p.att = off;   off += align_up(rows * c.D * es);
   p.u = off;     off += align_up(rows * size_t(c.mlp_hidden) * es);
-  p.h = off;     off += align_up(rrows * c.D * es);
+  p.hs = off;    off += align_up(rrows * c.D * sizeof(float));    // fp32 routed stream
   p.idx = off;   off += align_up(size_t(c.B) * c.L * sizeof(int32_t));
   p.score = off; off += align_up(rows * sizeof(float));
   p.total = off;
@@ -119,10 +114,12 @@ struct sr_handle {
   int32_t Kmax;
   Plan plan;
   bool trace = false;
+  bool fault_cleared = false;   // the fault word is zeroed by the first enqueuing call
   std::vector<TraceRec> pending;
   std::vector<cudaEvent_t> pool;
   sr_trace_entry acc[SR_KERN_COUNT] = {};
   void* at(size_t off) const { return ws + off; }
+  unsigned int* fault() const { return static_cast<unsigned int*>(at(plan.fault)); }
   ~sr_handle() {
     for (auto& r : pending) { cudaEventDestroy(r.ev0); cudaEventDestroy(r.ev1); }
     for (auto e : pool) cudaEventDestroy(e);
@@ -167,6 +164,7 @@ struct TraceScope {
 // GEMM and attention dispatch by dtype.
 cudaError_t gemm(const sr_handle* h, Epi epi, const void* A, const void* W, int M, int N, int K,
                  const sr::EpiArgs& ea, cudaStream_t s) {
+  if (h->dt == DType::BF16) return sr::launch_gemm_tc(epi, A, W, M, N, K, ea, s);
   return sr::launch_gemm_simt(h->dt, epi, A, W, M, N, K, ea, s);
 }
 
@@ -175,11 +173,12 @@ cudaError_t attention(const sr_handle* h, const void* qkv, void* out, int B, int
   return sr::launch_attention_simt(h->dt, qkv, out, B, T, h->cfg.heads, s);
 }
 
-// One pre-LN block (Sec. 3.3 Eq. 11) on the residual stream x [B*T, D], in place.
-// With `scatter` set this is the last sparse block: its FC2 epilogue writes
-// x0 + (h_out - h0) into the rows idx of `scatter_out` [B*Lx, D] instead of x.
-sr_status run_block(const sr_handle* hd, void* x, int B, int T, const sr_block_weights& w,
-                    bool scatter, void* scatter_out, const int32_t* idx, int Lx,
+// One pre-LN block (Sec. 3.3 Eq. 11) on the fp32 residual stream x [B*T, D], in
+// place.  With `scatter` set this is the last sparse block: its FC2 epilogue
+// writes x0 + (h_out - h0) into the rows idx of the stream `scatter_out`
+// [B*Lx, D] instead of x.
+sr_status run_block(const sr_handle* hd, float* x, int B, int T, const sr_block_weights& w,
+                    bool scatter, float* scatter_out, const int32_t* idx, int Lx,
                     cudaStream_t s) {
   const sr_config& c = hd->cfg;
   const int rows = B * T, D = c.D, H = c.mlp_hidden;
@@ -188,7 +187,7 @@ sr_status run_block(const sr_handle* hd, void* x, int B, int T, const sr_block_w
   void* qkv = hd->at(hd->plan.qkv);
   void* att = hd->at(hd->plan.att);
   void* u = hd->at(hd->plan.u);
-  const double ln_bytes = (2.0 * R * D + 2.0 * D) * es;
+  const double ln_bytes = R * D * (4.0 + es) + 2.0 * D * es;
   {
     TraceScope t(hd, SR_KERN_LAYERNORM, 0.0, ln_bytes, s);
     SR_CUDA(sr::launch_layernorm(hd->dt, x, w.ln1_g, w.ln1_b, ln, rows, D, c.ln_eps, s), "layernorm1");
@@ -196,7 +195,7 @@ sr_status run_block(const sr_handle* hd, void* x, int B, int T, const sr_block_w
   {
     TraceScope t(hd, SR_KERN_GEMM_QKV, 2.0 * R * 3 * D * D,
                  (R * D + 3.0 * D * D + R * 3 * D + 3.0 * D) * es, s);
-    sr::EpiArgs e1{w.bqkv, nullptr, qkv, nullptr, 0, 0};
+    sr::EpiArgs e1{w.bqkv, nullptr, qkv, nullptr, 0, 0, hd->fault()};
     SR_CUDA(gemm(hd, Epi::Bias, ln, w.wqkv, rows, 3 * D, D, e1, s), "qkv gemm");
   }
   {
@@ -205,8 +204,8 @@ sr_status run_block(const sr_handle* hd, void* x, int B, int T, const sr_block_w
     SR_CUDA(attention(hd, qkv, att, B, T, s), "attention");
   }
   {
-    TraceScope t(hd, SR_KERN_GEMM_OUT, 2.0 * R * D * D, (R * D + 1.0 * D * D + 2.0 * R * D + D) * es, s);
-    sr::EpiArgs e2{w.bo, x, x, nullptr, 0, 0};
+    TraceScope t(hd, SR_KERN_GEMM_OUT, 2.0 * R * D * D, (R * D + 1.0 * D * D + D) * es + 8.0 * R * D, s);
+    sr::EpiArgs e2{w.bo, x, x, nullptr, 0, 0, hd->fault()};
     SR_CUDA(gemm(hd, Epi::BiasResidual, att, w.wo, rows, D, D, e2, s), "out-proj gemm");
   }
   {
@@ -215,18 +214,18 @@ sr_status run_block(const sr_handle* hd, void* x, int B, int T, const sr_block_w
   }
   {
     TraceScope t(hd, SR_KERN_GEMM_FC1, 2.0 * R * H * D, (R * D + 1.0 * H * D + R * H + H) * es, s);
-    sr::EpiArgs e3{w.b1, nullptr, u, nullptr, 0, 0};
+    sr::EpiArgs e3{w.b1, nullptr, u, nullptr, 0, 0, hd->fault()};
     SR_CUDA(gemm(hd, Epi::BiasGelu, ln, w.w1, rows, H, D, e3, s), "fc1 gemm");
   }
   if (!scatter) {
-    TraceScope t(hd, SR_KERN_GEMM_FC2, 2.0 * R * D * H, (R * H + 1.0 * D * H + 2.0 * R * D + D) * es, s);
-    sr::EpiArgs e4{w.b2, x, x, nullptr, 0, 0};
+    TraceScope t(hd, SR_KERN_GEMM_FC2, 2.0 * R * D * H, (R * H + 1.0 * D * H + D) * es + 8.0 * R * D, s);
+    sr::EpiArgs e4{w.b2, x, x, nullptr, 0, 0, hd->fault()};
     SR_CUDA(gemm(hd, Epi::BiasResidual, u, w.w2, rows, D, H, e4, s), "fc2 gemm");
   } else {
     // reads h and x0 rows, writes the scattered rows, plus the index set
     TraceScope t(hd, SR_KERN_GEMM_FC2_SCATTER, 2.0 * R * D * H,
-                 (R * H + 1.0 * D * H + 3.0 * R * D + D) * es + 4.0 * R, s);
-    sr::EpiArgs e4{w.b2, x, scatter_out, idx, T, Lx};
+                 (R * H + 1.0 * D * H + D) * es + 12.0 * R * D + 4.0 * R, s);
+    sr::EpiArgs e4{w.b2, x, scatter_out, idx, T, Lx, hd->fault()};
     SR_CUDA(gemm(hd, Epi::BiasResidualScatter, u, w.w2, rows, D, H, e4, s), "fc2 scatter gemm");
   }
   return SR_OK;
@@ -240,7 +239,7 @@ bool weights_ok(const sr_block_weights& w) {
   return true;
 }
 
-sr_status do_select(sr_handle* h, const void* x, int32_t K, uint64_t seed, int32_t* idx,
+sr_status do_select(sr_handle* h, const float* x, int32_t K, uint64_t seed, int32_t* idx,
                     cudaStream_t s) {
   const sr_config& c = h->cfg;
   const double sel_bytes = 4.0 * c.B * K +
@@ -282,7 +281,7 @@ sr_status sr_create(const sr_config* cfg, void* workspace, size_t ws_bytes, sr_h
   if (ws_bytes < full.total) {
     const Plan none = make_plan(*cfg, 0);
     if (ws_bytes < none.total) return fail(SR_ERR_WORKSPACE, "workspace too small");
-    const size_t per_row = size_t(cfg->B) * cfg->D * elem_size(cfg->dtype);
+    const size_t per_row = size_t(cfg->B) * cfg->D * sizeof(float);
     Kmax = int32_t((ws_bytes - none.total) / (per_row ? per_row : 1));
     while (Kmax > 0 && make_plan(*cfg, Kmax).total > ws_bytes) --Kmax;
     if (Kmax < 1) return fail(SR_ERR_WORKSPACE, "workspace too small for any routed token");
@@ -315,7 +314,14 @@ sr_status sr_select(sr_handle* h, const void* x, float keep_ratio, uint64_t seed
   if (h->cfg.selector == SR_SEL_TOPK_L2 && (!x || !aligned(x, 16)))
     return fail(SR_ERR_INVALID_ARG, "top-K selection needs a 16-byte aligned x");
   if (K_out) *K_out = K;
-  return do_select(h, x, K, seed, idx, static_cast<cudaStream_t>(stream));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  float* xs = nullptr;
+  if (h->cfg.selector == SR_SEL_TOPK_L2) {
+    // the norms are taken of the stored activations: widen them into the stream buffer
+    xs = static_cast<float*>(h->at(h->plan.xs));
+    SR_CUDA(sr::launch_widen(h->dt, x, xs, size_t(h->cfg.B) * h->cfg.L * h->cfg.D, s), "widen x");
+  }
+  return do_select(h, xs, K, seed, idx, s);
 }
 
 sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, float keep_ratio,
@@ -340,35 +346,46 @@ sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, flo
   if (xb != ob && xb < ob + bytes && ob < xb + bytes)
     return fail(SR_ERR_INVALID_ARG, "out partially overlaps x");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (xb != ob) {
-    TraceScope t(h, SR_KERN_COPY, 0.0, 2.0 * bytes, s);
-    SR_CUDA(cudaMemcpyAsync(out, x, bytes, cudaMemcpyDeviceToDevice, s), "copy x -> out");
+  if (!h->fault_cleared) {
+    SR_CUDA(cudaMemsetAsync(h->fault(), 0, sizeof(unsigned int), s), "clear fault word");
+    h->fault_cleared = true;
+  }
+  const size_t n = size_t(c.B) * c.L * c.D;
+  float* xs = static_cast<float*>(h->at(h->plan.xs));
+  {
+    // the residual stream is held in fp32 for the whole forward
+    TraceScope t(h, SR_KERN_COPY, 0.0, double(bytes) + 4.0 * n, s);
+    SR_CUDA(sr::launch_widen(h->dt, x, xs, n, s), "widen x");
   }
   sr_status st;
   // stage 1: dense early
   for (int i = 0; i < c.n1; ++i)
-    if ((st = run_block(h, out, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
+    if ((st = run_block(h, xs, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
   int32_t* idx = idx_out ? idx_out : static_cast<int32_t*>(h->at(h->plan.idx));
   if (route || idx_out)
-    if ((st = do_select(h, out, K, seed, idx, s)) != SR_OK) return st;
+    if ((st = do_select(h, xs, K, seed, idx, s)) != SR_OK) return st;
   if (route) {
     // stage 2: gather, sparse middle, delta scatter in the last block's epilogue
-    void* hbuf = h->at(h->plan.h);
+    float* hs = static_cast<float*>(h->at(h->plan.hs));
     {
-      TraceScope t(h, SR_KERN_GATHER, 0.0, 2.0 * c.B * K * c.D * h->es + 4.0 * c.B * K, s);
-      SR_CUDA(sr::launch_gather_rows(h->dt, out, idx, c.B, c.L, K, c.D, hbuf, s), "gather");
+      TraceScope t(h, SR_KERN_GATHER, 0.0, 8.0 * c.B * K * c.D + 4.0 * c.B * K, s);
+      SR_CUDA(sr::launch_gather_rows(xs, idx, c.B, c.L, K, c.D, hs, s), "gather");
     }
     for (int i = c.n1; i < c.n1 + c.n2; ++i) {
       const bool last = i == c.n1 + c.n2 - 1;
-      if ((st = run_block(h, hbuf, c.B, K, w[i], last, out, idx, c.L, s)) != SR_OK) return st;
+      if ((st = run_block(h, hs, c.B, K, w[i], last, xs, idx, c.L, s)) != SR_OK) return st;
     }
   } else {
     for (int i = c.n1; i < c.n1 + c.n2; ++i)
-      if ((st = run_block(h, out, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
+      if ((st = run_block(h, xs, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
   }
   // stage 3: dense late
   for (int i = c.n1 + c.n2; i < N; ++i)
-    if ((st = run_block(h, out, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
+    if ((st = run_block(h, xs, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
+  {
+    TraceScope t(h, SR_KERN_COPY, 0.0, double(bytes) + 4.0 * n, s);
+    SR_CUDA(sr::launch_narrow(h->dt, xs, out, n, s), "narrow out");
+  }
   return SR_OK;
 }
 
@@ -426,5 +443,16 @@ const char* sr_status_string(sr_status s) {
 }
 
 const char* sr_last_error_message(void) { return g_last_msg.c_str(); }
+
+sr_status sr_device_fault(sr_handle* h, uint32_t* fault, int clear, void* stream) {
+  if (!h || !fault) return fail(SR_ERR_INVALID_ARG, "handle or fault is NULL");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unsigned int f = 0;
+  SR_CUDA(cudaMemcpyAsync(&f, h->fault(), sizeof(f), cudaMemcpyDeviceToHost, s), "read fault word");
+  SR_CUDA(cudaStreamSynchronize(s), "stream synchronize");
+  if (clear) SR_CUDA(cudaMemsetAsync(h->fault(), 0, sizeof(f), s), "clear fault word");
+  *fault = f;
+  return SR_OK;
+}
 
 }  // extern "C"

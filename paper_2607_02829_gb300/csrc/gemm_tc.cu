@@ -1,0 +1,306 @@
+// tcgen05 GEMM for the bf16 block projections: C[M, N] = A[M, K] B[N, K]^T with
+// the block's epilogues fused (bias; bias + GELU; bias + fp32 residual add; bias
+// + residual + the delta scatter of Eq. 9 for the last sparse block).
+//
+// Persistent, warp-specialised, one CTA per SM (192 threads):
+//   warp 0      TMA producer: A and B tiles (128 x 64 and BN x 64 bf16, 128-byte
+//               swizzle) into a ring of shared-memory stages;
+//   warp 1      owns the tensor memory and issues tcgen05.mma (M = 128, N = BN,
+//               K = 16) into one of two TMEM accumulators;
+//   warps 2..5  epilogue: tcgen05.ld of the finished accumulator (one row per
+//               thread), the fused epilogue, global stores; the second
+//               accumulator lets the next tile's MMAs run meanwhile.
+// Rows beyond M are zero-filled by TMA and never stored.  Requires K % 64 == 0
+// and N % BN == 0 (checked by the launcher).
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc_ptx.cuh"
+
+namespace sr {
+namespace {
+
+using namespace tc;
+
+constexpr int BM = 128, BK = 64;
+constexpr int kThreads = 192;
+constexpr int kEpiThreads = 128;
+
+template <int BN>
+struct GemmCfg {
+  static constexpr int kStages = BN == 256 ? 4 : 6;
+  static constexpr int kABytes = BM * BK * 2;        // 16 KB
+  static constexpr int kBBytes = BN * BK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kTmemCols = 2 * BN;           // two accumulators
+  static constexpr size_t kSmem = size_t(kStages) * kStageBytes + 1024 /*align*/ + 256 /*bars*/;
+};
+
+struct Smem {
+  uint64_t full[8], empty[8], tfull[2], tempty[2], drain;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Epilogue of 32 consecutive columns n..n+31 of row m (acc in fp32 bits).
+template <Epi E>
+__device__ __forceinline__ void epilogue32(const EpiArgs& ea, int m, int n, int N,
+                                           const uint32_t (&acc)[32]) {
+  const uint4* bias4 = reinterpret_cast<const uint4*>(static_cast<const bf16*>(ea.bias) + n);
+  float v[32];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint4 bq = __ldg(bias4 + q);
+    const uint32_t bw[4] = {bq.x, bq.y, bq.z, bq.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      v[8 * q + 2 * j] = __uint_as_float(acc[8 * q + 2 * j]) + bf16_lo(bw[j]);
+      v[8 * q + 2 * j + 1] = __uint_as_float(acc[8 * q + 2 * j + 1]) + bf16_hi(bw[j]);
+    }
+  }
+  if constexpr (E == Epi::Bias || E == Epi::BiasGelu) {
+    if constexpr (E == Epi::BiasGelu) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = gelu_erf(v[j]);
+    }
+    uint4* o = reinterpret_cast<uint4*>(static_cast<bf16*>(ea.out) + size_t(m) * N + n);
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      o[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                        pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+  } else {
+    const float4* r = reinterpret_cast<const float4*>(ea.res + size_t(m) * N + n);
+    float4 rv[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) rv[q] = r[q];
+    if constexpr (E == Epi::BiasResidual) {
+      float4* o = reinterpret_cast<float4*>(static_cast<float*>(ea.out) + size_t(m) * N + n);
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        o[q] = make_float4(rv[q].x + v[4 * q], rv[q].y + v[4 * q + 1], rv[q].z + v[4 * q + 2],
+                           rv[q].w + v[4 * q + 3]);
+    } else {
+      // last sparse block: hn = h + f(h); x'[xrow] = x0 + (hn - h0), h0 == x0
+      const int b = m / ea.Kr;
+      const size_t xrow = size_t(b) * ea.Lx + ea.idx[m];
+      float4* o = reinterpret_cast<float4*>(static_cast<float*>(ea.out) + xrow * N + n);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const float4 x0 = o[q];
+        const float hn[4] = {rv[q].x + v[4 * q], rv[q].y + v[4 * q + 1], rv[q].z + v[4 * q + 2],
+                             rv[q].w + v[4 * q + 3]};
+        o[q] = make_float4(x0.x + (hn[0] - x0.x), x0.y + (hn[1] - x0.y), x0.z + (hn[2] - x0.z),
+                           x0.w + (hn[3] - x0.w));
+      }
+    }
+  }
+}
+
+template <int BN, Epi E>
+__global__ void __launch_bounds__(kThreads, 1)
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+               int M, int N, int K, EpiArgs ea) {
+  using C = GemmCfg<BN>;
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* base = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  unsigned char* sA = base;
+  unsigned char* sB = base + size_t(C::kStages) * C::kABytes;
+  Smem* sm = reinterpret_cast<Smem*>(base + size_t(C::kStages) * C::kStageBytes);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m_tiles = (M + BM - 1) / BM;
+  const int n_tiles = N / BN;
+  const int tiles = m_tiles * n_tiles;
+  const int kblocks = K / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) { mbar_init(&sm->full[s], 1); mbar_init(&sm->empty[s], 1); }
+    for (int a = 0; a < 2; ++a) { mbar_init(&sm->tfull[a], 1); mbar_init(&sm->tempty[a], kEpiThreads); }
+    mbar_init(&sm->drain, 1);
+    sm->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) { prefetch_tmap(&tmA); prefetch_tmap(&tmB); }
+  if (warp == 1) tmem_alloc(&sm->tmem_base, C::kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm->tmem_base;
+  volatile int* abort = &sm->abort;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued = 0, issued_phase = 0;    // per stage: loads in flight, their parity
+      for (int t = blockIdx.x; t < tiles && !*abort; t += gridDim.x) {
+        const int mt = t % m_tiles, nt = t / m_tiles;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&sm->empty[stage], phase ^ 1, abort, ea.fault)) break;
+          mbar_arrive_expect_tx(&sm->full[stage], C::kStageBytes);
+          tma_load_2d(&tmA, sA + size_t(stage) * C::kABytes, &sm->full[stage], kb * BK, mt * BM);
+          tma_load_2d(&tmB, sB + size_t(stage) * C::kBBytes, &sm->full[stage], kb * BK, nt * BN);
+          issued |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == C::kStages) { stage = 0; phase ^= 1; }
+        }
+      }
+      // every load this thread issued lands before the CTA may exit (immediate
+      // unless an aborted pipeline left loads unconsumed)
+      int no_abort = 0;
+      for (int st = 0; st < C::kStages; ++st)
+        if (issued & (1u << st)) mbar_wait(&sm->full[st], (issued_phase >> st) & 1u, &no_abort, ea.fault);
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16(BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      for (int t = blockIdx.x; t < tiles && !*abort; t += gridDim.x, ++it) {
+        const int acc = it & 1;
+        const uint32_t aphase = (it >> 1) & 1;
+        if (!mbar_wait(&sm->tempty[acc], aphase ^ 1, abort, ea.fault)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + uint32_t(acc * BN);
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&sm->full[stage], phase, abort, ea.fault)) break;
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + size_t(stage) * C::kABytes);
+          const uint32_t b0 = smem_u32(sB + size_t(stage) * C::kBBytes);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            mma_bf16(d, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc,
+                     (kb | k) != 0 ? 1u : 0u);
+          mma_commit(&sm->empty[stage]);
+          if (++stage == C::kStages) { stage = 0; phase ^= 1; }
+        }
+        mma_commit(&sm->tfull[acc]);
+      }
+      // every MMA issued has completed before the tensor memory is released
+      int no_abort = 0;
+      mma_commit(&sm->drain);
+      mbar_wait(&sm->drain, 0, &no_abort, ea.fault);
+    }
+  } else {
+    // ---------------------------------------------------------- epilogue
+    const int q = warp & 3;                 // TMEM lane quarter of this warp
+    const int row = q * 32 + lane;
+    int it = 0;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++it) {
+      const int mt = t % m_tiles, nt = t / m_tiles;
+      const int acc = it & 1;
+      const uint32_t aphase = (it >> 1) & 1;
+      if (!mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault)) break;
+      tc_fence_after();
+      const int m = mt * BM + row;
+      const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        uint32_t r[32];
+        tmem_ld32(tbase + uint32_t(c), r);
+        tmem_wait_ld();
+        if (m < M) epilogue32<E>(ea, m, nt * BN + c, N, r);
+      }
+      tc_fence_before();
+      mbar_arrive(&sm->tempty[acc]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+cudaError_t get_encoder() {
+  if (g_encode) return cudaSuccess;
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                   cudaEnableDefault, &q);
+  if (e != cudaSuccess) return e;
+  if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+  g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  return cudaSuccess;
+}
+
+// 2-D bf16 tensor map over a row-major [rows, cols] matrix, box [box_rows, 64].
+cudaError_t make_map_2d(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols,
+                        uint32_t box_rows) {
+  cudaError_t e = get_encoder();
+  if (e != cudaSuccess) return e;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+int g_num_sms = 0;
+
+template <int BN, Epi E>
+cudaError_t launch_bn(const void* A, const void* W, int M, int N, int K, const EpiArgs& ea,
+                      cudaStream_t s) {
+  using C = GemmCfg<BN>;
+  CUtensorMap ta, tb;
+  cudaError_t e = make_map_2d(&ta, A, uint64_t(M), uint64_t(K), BM);
+  if (e != cudaSuccess) return e;
+  e = make_map_2d(&tb, W, uint64_t(N), uint64_t(K), BN);
+  if (e != cudaSuccess) return e;
+  static bool attr_set = false;
+  if (!attr_set) {
+    e = cudaFuncSetAttribute(gemm_tc_kernel<BN, E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             int(C::kSmem));
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  if (g_num_sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+  }
+  const int tiles = ((M + BM - 1) / BM) * (N / BN);
+  const int grid = tiles < g_num_sms ? tiles : g_num_sms;
+  gemm_tc_kernel<BN, E><<<grid, kThreads, C::kSmem, s>>>(ta, tb, M, N, K, ea);
+  return cudaGetLastError();
+}
+
+template <int BN>
+cudaError_t launch_epi(Epi epi, const void* A, const void* W, int M, int N, int K,
+                       const EpiArgs& ea, cudaStream_t s) {
+  switch (epi) {
+    case Epi::Bias: return launch_bn<BN, Epi::Bias>(A, W, M, N, K, ea, s);
+    case Epi::BiasGelu: return launch_bn<BN, Epi::BiasGelu>(A, W, M, N, K, ea, s);
+    case Epi::BiasResidual: return launch_bn<BN, Epi::BiasResidual>(A, W, M, N, K, ea, s);
+    case Epi::BiasResidualScatter: return launch_bn<BN, Epi::BiasResidualScatter>(A, W, M, N, K, ea, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* W, int M, int N, int K,
+                           const EpiArgs& ea, cudaStream_t s) {
+  if (M < 1 || K % BK != 0 || N % 64 != 0) return cudaErrorInvalidValue;
+  if (N % 256 == 0) return launch_epi<256>(epi, A, W, M, N, K, ea, s);
+  if (N % 128 == 0) return launch_epi<128>(epi, A, W, M, N, K, ea, s);
+  return launch_epi<64>(epi, A, W, M, N, K, ea, s);
+}
+
+}  // namespace sr

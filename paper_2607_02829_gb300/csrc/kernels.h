@@ -14,8 +14,10 @@ enum class DType : int { F32 = 0, BF16 = 1 };
 // Random: K smallest SplitMix64 keys per sample (ties by index), sorted indices.
 cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared,
                                  int32_t* idx, cudaStream_t s);
-// Squared L2 norm of every token of x [B*L, D] into score [B*L] (fp32).
-cudaError_t launch_token_sq_norms(DType dt, const void* x, int rows, int D, float* score,
+// Squared L2 norm of every token of the fp32 stream x [B*L, D] into score [B*L];
+// each value is first rounded to the storage dtype dt (the activation the model
+// stores), its square accumulated in fp32.
+cudaError_t launch_token_sq_norms(DType dt, const float* x, int rows, int D, float* score,
                                   cudaStream_t s);
 // K largest scores per sample (ties to the lower index), sorted indices.
 cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t* idx,
@@ -23,37 +25,50 @@ cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t*
 // Largest L the one-CTA-per-sample selection kernels accept (keys in shared memory).
 int select_max_L();
 
-// ---- gather (Eq. 8): h[b*K + k, :] = x[b*L + idx[b*K + k], :] ------------
-cudaError_t launch_gather_rows(DType dt, const void* x, const int32_t* idx, int B, int L, int K,
-                               int D, void* h, cudaStream_t s);
+// ---- gather (Eq. 8) on the fp32 stream: h[b*K + k, :] = x[b*L + idx[b*K + k], :]
+cudaError_t launch_gather_rows(const float* x, const int32_t* idx, int B, int L, int K, int D,
+                               float* h, cudaStream_t s);
 
-// ---- LayerNorm over D: y = (x - mean) / sqrt(var + eps) * g + b -----------
-cudaError_t launch_layernorm(DType dt, const void* x, const void* g, const void* b, void* y,
+// ---- storage dtype <-> fp32 residual stream, n elements (n % 8 == 0) ------
+cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream_t s);
+cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStream_t s);
+
+// ---- LayerNorm over D from the fp32 stream into the storage dtype ---------
+//      y = (x - mean) / sqrt(var + eps) * g + b
+cudaError_t launch_layernorm(DType dt, const float* x, const void* g, const void* b, void* y,
                              int rows, int D, float eps, cudaStream_t s);
 
 // ---- GEMM C = A B^T with fused epilogues ---------------------------------
-// A [M, K] row-major, B [N, K] row-major (nn.Linear weight), fp32 accumulate.
+// A [M, K] row-major, B [N, K] row-major (nn.Linear weight), both in the storage
+// dtype, fp32 accumulate.  Bias is in the storage dtype.
 enum class Epi : int {
-  Bias = 0,          // out[m, n] = acc + bias[n]
-  BiasGelu = 1,      // out[m, n] = GELU(acc + bias[n])
-  BiasResidual = 2,  // out[m, n] = res[m, n] + acc + bias[n]        (out may == res)
-  BiasResidualScatter = 3,  // hn = res[m, n] + acc + bias[n]; row m = b*Kr + k maps to
-                            // xrow = b*Lx + idx[m]; out[xrow, n] = x0 + (hn - x0), x0 = out[xrow, n]
+  Bias = 0,          // out[m, n] = acc + bias[n]                   (out: storage dtype)
+  BiasGelu = 1,      // out[m, n] = GELU(acc + bias[n])             (out: storage dtype)
+  BiasResidual = 2,  // out[m, n] = res[m, n] + acc + bias[n]       (fp32 stream, out may == res)
+  BiasResidualScatter = 3,  // hn = res[m, n] + acc + bias[n] (fp32 routed stream); row
+                            // m = b*Kr + k maps to xrow = b*Lx + idx[m]; the fp32 stream
+                            // out[xrow, n] = x0 + (hn - x0) with x0 = out[xrow, n]
 };
 struct EpiArgs {
   const void* bias;     // [N]
-  const void* res;      // [M, N] (BiasResidual*)
-  void* out;            // [M, N], or [B*Lx, N] for the scatter epilogue
+  const float* res;     // [M, N] fp32 stream (BiasResidual*)
+  void* out;            // [M, N], or the fp32 stream [B*Lx, N] for the scatter epilogue
   const int32_t* idx;   // [M] for the scatter epilogue
   int Kr;               // routed rows per sample (scatter)
   int Lx;               // tokens per sample of the scatter target
+  unsigned int* fault;  // fault word (bit 0: a bounded barrier wait timed out)
 };
-cudaError_t launch_gemm(DType dt, Epi epi, const void* A, const void* Bw, int M, int N, int K,
-                        const EpiArgs& ea, cudaStream_t s);
+// CUDA-core GEMM (fp32 storage) and tcgen05 GEMM (bf16 storage; K % 64 == 0,
+// N % 64 == 0).
+cudaError_t launch_gemm_simt(DType dt, Epi epi, const void* A, const void* Bw, int M, int N,
+                             int K, const EpiArgs& ea, cudaStream_t s);
+cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* Bw, int M, int N, int K,
+                           const EpiArgs& ea, cudaStream_t s);
+
 
 // ---- attention core: per (sample, head) softmax(q k^T / sqrt(64)) v ------
 // qkv [B*T, 3D] (q | k | v, head h at columns 64h..64h+63 of each); out [B*T, D].
-cudaError_t launch_attention(DType dt, const void* qkv, void* out, int B, int T, int heads,
-                             cudaStream_t s);
+cudaError_t launch_attention_simt(DType dt, const void* qkv, void* out, int B, int T, int heads,
+                                  cudaStream_t s);
 
 }  // namespace sr

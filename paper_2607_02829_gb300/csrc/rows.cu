@@ -1,18 +1,20 @@
-// Row-wise HBM-bound kernels: the routed-token gather (Eq. 8) and LayerNorm
-// (the LN of the pre-LN block, Sec. 3.3 Eq. 11).  One warp owns one row; rows
-// move as 16-byte vectors, all loads of a row are issued before any use.
+// Row-wise HBM-bound kernels on the fp32 residual stream: the routed-token
+// gather (Eq. 8), LayerNorm (the LN of the pre-LN block, Sec. 3.3 Eq. 11) and
+// the conversions between the caller's storage dtype and the stream.  One warp
+// owns one row; rows move as 16-byte vectors, all loads of a row are issued
+// before any use.
 #include "common.cuh"
 #include "kernels.h"
 
 namespace sr {
 namespace {
 
-// h[b*K + k, :] = x[b*L + idx[b*K + k], :]  -- a bit copy of D * sizeof(T) bytes.
-template <typename T, int NV>
+// h[b*K + k, :] = x[b*L + idx[b*K + k], :]  -- a bit copy of D fp32 values.
+template <int NV>
 __global__ void __launch_bounds__(256)
-gather_rows_kernel(const T* __restrict__ x, const int32_t* __restrict__ idx, int L, int K,
-                   int D, int rows, T* __restrict__ h) {
-  constexpr int V = Elem<T>::kVec;
+gather_rows_kernel(const float* __restrict__ x, const int32_t* __restrict__ idx, int L, int K,
+                   int D, int rows, float* __restrict__ h) {
+  constexpr int V = 4;
   const int lane = threadIdx.x & 31;
   const int nv = D / V;
   const int warps = (gridDim.x * blockDim.x) >> 5;
@@ -31,29 +33,36 @@ gather_rows_kernel(const T* __restrict__ x, const int32_t* __restrict__ idx, int
   }
 }
 
-// y = (x - mean) / sqrt(var + eps) * g + b, statistics in fp32, two passes over
-// the row held in registers (biased variance).
+// y = (x - mean) / sqrt(var + eps) * g + b from the fp32 stream x into the
+// storage dtype T, statistics in fp32, two passes over the row held in
+// registers (biased variance).  Rows are read as 4-float vectors, g, b and y
+// move as 16-byte vectors of T.
 template <typename T, int NV>
 __global__ void __launch_bounds__(256)
-layernorm_kernel(const T* __restrict__ x, const T* __restrict__ g, const T* __restrict__ bta,
+layernorm_kernel(const float* __restrict__ x, const T* __restrict__ g, const T* __restrict__ bta,
                  T* __restrict__ y, int rows, int D, float eps) {
   constexpr int V = Elem<T>::kVec;
   const int lane = threadIdx.x & 31;
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   if (row >= rows) return;
   const int nv = D / V;
-  const uint4* xr = reinterpret_cast<const uint4*>(x + size_t(row) * D);
+  const float4* xr = reinterpret_cast<const float4*>(x + size_t(row) * D);
   float f[NV][V];
   float sum = 0.f;
 #pragma unroll
   for (int j = 0; j < NV; ++j) {
     if (lane + 32 * j < nv) {
-      unpack16(__ldg(xr + lane + 32 * j), f[j]);
+#pragma unroll
+      for (int q = 0; q < V / 4; ++q) {
+        const float4 v4 = __ldg(xr + (lane + 32 * j) * (V / 4) + q);
+        f[j][4 * q] = v4.x; f[j][4 * q + 1] = v4.y; f[j][4 * q + 2] = v4.z; f[j][4 * q + 3] = v4.w;
+      }
 #pragma unroll
       for (int e = 0; e < V; ++e) sum += f[j][e];
     }
   }
-  const float mean = warp_sum(sum) / float(D);
+  const float inv_d = 1.0f / float(D);
+  const float mean = warp_sum(sum) * inv_d;
   float sq = 0.f;
 #pragma unroll
   for (int j = 0; j < NV; ++j) {
@@ -62,7 +71,7 @@ layernorm_kernel(const T* __restrict__ x, const T* __restrict__ g, const T* __re
       for (int e = 0; e < V; ++e) { const float c = f[j][e] - mean; sq = fmaf(c, c, sq); }
     }
   }
-  const float rstd = rsqrtf(warp_sum(sq) / float(D) + eps);
+  const float rstd = rsqrtf(warp_sum(sq) * inv_d + eps);
   const uint4* gr = reinterpret_cast<const uint4*>(g);
   const uint4* br = reinterpret_cast<const uint4*>(bta);
   uint4* yr = reinterpret_cast<uint4*>(y + size_t(row) * D);
@@ -80,22 +89,58 @@ layernorm_kernel(const T* __restrict__ x, const T* __restrict__ g, const T* __re
   }
 }
 
-template <typename T, int NV>
-cudaError_t gather_t(const void* x, const int32_t* idx, int B, int L, int K, int D, void* h,
+template <int NV>
+cudaError_t gather_t(const float* x, const int32_t* idx, int B, int L, int K, int D, float* h,
                      cudaStream_t s) {
   const int rows = B * K;
   int blocks = (rows + 7) / 8;
   if (blocks > 152 * 16) blocks = 152 * 16;
-  gather_rows_kernel<T, NV><<<blocks, 256, 0, s>>>(static_cast<const T*>(x), idx, L, K, D, rows,
-                                                   static_cast<T*>(h));
+  gather_rows_kernel<NV><<<blocks, 256, 0, s>>>(x, idx, L, K, D, rows, h);
   return cudaGetLastError();
 }
 
+// Storage dtype <-> fp32 stream, n elements (n % 8 == 0), 16-byte vectors.
+template <typename T>
+__global__ void __launch_bounds__(256)
+widen_kernel(const T* __restrict__ x, float* __restrict__ y, size_t nvec) {
+  constexpr int V = Elem<T>::kVec;
+  for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
+       i += size_t(gridDim.x) * blockDim.x) {
+    float f[V];
+    unpack16(__ldg(reinterpret_cast<const uint4*>(x) + i), f);
+    float4* o = reinterpret_cast<float4*>(y) + i * (V / 4);
+#pragma unroll
+    for (int q = 0; q < V / 4; ++q) o[q] = make_float4(f[4 * q], f[4 * q + 1], f[4 * q + 2], f[4 * q + 3]);
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256)
+narrow_kernel(const float* __restrict__ x, T* __restrict__ y, size_t nvec) {
+  constexpr int V = Elem<T>::kVec;
+  for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
+       i += size_t(gridDim.x) * blockDim.x) {
+    float f[V];
+    const float4* in = reinterpret_cast<const float4*>(x) + i * (V / 4);
+#pragma unroll
+    for (int q = 0; q < V / 4; ++q) {
+      const float4 v4 = __ldg(in + q);
+      f[4 * q] = v4.x; f[4 * q + 1] = v4.y; f[4 * q + 2] = v4.z; f[4 * q + 3] = v4.w;
+    }
+    reinterpret_cast<uint4*>(y)[i] = pack16(f);
+  }
+}
+
+int grid_for(size_t nvec) {
+  size_t b = (nvec + 255) / 256;
+  return int(b < 152 * 32 ? b : 152 * 32);
+}
+
 template <typename T, int NV>
-cudaError_t layernorm_t(const void* x, const void* g, const void* b, void* y, int rows, int D,
+cudaError_t layernorm_t(const float* x, const void* g, const void* b, void* y, int rows, int D,
                         float eps, cudaStream_t s) {
   layernorm_kernel<T, NV><<<(rows + 7) / 8, 256, 0, s>>>(
-      static_cast<const T*>(x), static_cast<const T*>(g), static_cast<const T*>(b),
+      x, static_cast<const T*>(g), static_cast<const T*>(b),
       static_cast<T*>(y), rows, D, eps);
   return cudaGetLastError();
 }
@@ -105,25 +150,40 @@ template <typename T> int lanes_nv(int D) { return (D / Elem<T>::kVec + 31) / 32
 
 }  // namespace
 
-cudaError_t launch_gather_rows(DType dt, const void* x, const int32_t* idx, int B, int L, int K,
-                               int D, void* h, cudaStream_t s) {
-  if (dt == DType::BF16) {
-    const int nv = lanes_nv<bf16>(D);
-    if (nv <= 1) return gather_t<bf16, 1>(x, idx, B, L, K, D, h, s);
-    if (nv <= 2) return gather_t<bf16, 2>(x, idx, B, L, K, D, h, s);
-    if (nv <= 4) return gather_t<bf16, 4>(x, idx, B, L, K, D, h, s);
-    if (nv <= 8) return gather_t<bf16, 8>(x, idx, B, L, K, D, h, s);
-  } else {
-    const int nv = lanes_nv<float>(D);
-    if (nv <= 1) return gather_t<float, 1>(x, idx, B, L, K, D, h, s);
-    if (nv <= 2) return gather_t<float, 2>(x, idx, B, L, K, D, h, s);
-    if (nv <= 4) return gather_t<float, 4>(x, idx, B, L, K, D, h, s);
-    if (nv <= 8) return gather_t<float, 8>(x, idx, B, L, K, D, h, s);
-  }
+cudaError_t launch_gather_rows(const float* x, const int32_t* idx, int B, int L, int K, int D,
+                               float* h, cudaStream_t s) {
+  const int nv = lanes_nv<float>(D);
+  if (nv <= 1) return gather_t<1>(x, idx, B, L, K, D, h, s);
+  if (nv <= 2) return gather_t<2>(x, idx, B, L, K, D, h, s);
+  if (nv <= 4) return gather_t<4>(x, idx, B, L, K, D, h, s);
+  if (nv <= 8) return gather_t<8>(x, idx, B, L, K, D, h, s);
+  if (nv <= 16) return gather_t<16>(x, idx, B, L, K, D, h, s);
   return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_layernorm(DType dt, const void* x, const void* g, const void* b, void* y,
+cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream_t s) {
+  if (dt == DType::BF16) {
+    const size_t nvec = n / 8;
+    widen_kernel<bf16><<<grid_for(nvec), 256, 0, s>>>(static_cast<const bf16*>(x), y, nvec);
+  } else {
+    const size_t nvec = n / 4;
+    widen_kernel<float><<<grid_for(nvec), 256, 0, s>>>(static_cast<const float*>(x), y, nvec);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStream_t s) {
+  if (dt == DType::BF16) {
+    const size_t nvec = n / 8;
+    narrow_kernel<bf16><<<grid_for(nvec), 256, 0, s>>>(x, static_cast<bf16*>(y), nvec);
+  } else {
+    const size_t nvec = n / 4;
+    narrow_kernel<float><<<grid_for(nvec), 256, 0, s>>>(x, static_cast<float*>(y), nvec);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_layernorm(DType dt, const float* x, const void* g, const void* b, void* y,
                              int rows, int D, float eps, cudaStream_t s) {
   if (dt == DType::BF16) {
     const int nv = lanes_nv<bf16>(D);

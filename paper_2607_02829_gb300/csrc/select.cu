@@ -153,22 +153,25 @@ select_topk_kernel(int L, int K, const float* __restrict__ score, int32_t* idx) 
   select_smallest_sorted<uint32_t>(keys, L, K, idx + size_t(b) * K);
 }
 
-// One warp per token: fp32 sum of squares over D, 16-byte loads.
+// One warp per token: every fp32 stream value is rounded to the storage dtype T
+// (the activation as the model stores it), then squared and summed in fp32.
 template <typename T>
 __global__ void __launch_bounds__(256)
-token_sq_norms_kernel(const T* __restrict__ x, int rows, int D, float* __restrict__ score) {
-  constexpr int V = Elem<T>::kVec;
+token_sq_norms_kernel(const float* __restrict__ x, int rows, int D, float* __restrict__ score) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= rows) return;
-  const uint4* row = reinterpret_cast<const uint4*>(x + size_t(warp) * D);
-  const int nv = D / V;
+  const float4* row = reinterpret_cast<const float4*>(x + size_t(warp) * D);
+  const int nv = D / 4;
   float acc = 0.f;
   for (int v = lane; v < nv; v += 32) {
-    float f[V];
-    unpack16(__ldg(row + v), f);
+    const float4 q = __ldg(row + v);
+    const float f[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
-    for (int j = 0; j < V; ++j) acc = fmaf(f[j], f[j], acc);
+    for (int j = 0; j < 4; ++j) {
+      const float r = Elem<T>::to_f(Elem<T>::from_f(f[j]));
+      acc = fmaf(r, r, acc);
+    }
   }
   acc = warp_sum(acc);
   if (lane == 0) score[warp] = acc;
@@ -198,13 +201,13 @@ cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t*
   return cudaGetLastError();
 }
 
-cudaError_t launch_token_sq_norms(DType dt, const void* x, int rows, int D, float* score,
+cudaError_t launch_token_sq_norms(DType dt, const float* x, int rows, int D, float* score,
                                   cudaStream_t s) {
   const int blocks = (rows + 7) / 8;
   if (dt == DType::BF16)
-    token_sq_norms_kernel<bf16><<<blocks, 256, 0, s>>>(static_cast<const bf16*>(x), rows, D, score);
+    token_sq_norms_kernel<bf16><<<blocks, 256, 0, s>>>(x, rows, D, score);
   else
-    token_sq_norms_kernel<float><<<blocks, 256, 0, s>>>(static_cast<const float*>(x), rows, D, score);
+    token_sq_norms_kernel<float><<<blocks, 256, 0, s>>>(x, rows, D, score);
   return cudaGetLastError();
 }
 

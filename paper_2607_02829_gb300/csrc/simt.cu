@@ -21,17 +21,17 @@ __device__ __forceinline__ void epilogue_store(const EpiArgs& ea, int m, int n, 
   } else if constexpr (E == Epi::BiasGelu) {
     static_cast<T*>(ea.out)[size_t(m) * N + n] = Elem<T>::from_f(gelu_erf(v));
   } else if constexpr (E == Epi::BiasResidual) {
-    const float r = Elem<T>::to_f(static_cast<const T*>(ea.res)[size_t(m) * N + n]);
-    static_cast<T*>(ea.out)[size_t(m) * N + n] = Elem<T>::from_f(r + v);
+    const float r = ea.res[size_t(m) * N + n];
+    static_cast<float*>(ea.out)[size_t(m) * N + n] = r + v;
   } else {
     // last sparse block: hn = h + f(h); x'[xrow] = x0 + (hn - h0), h0 == x0
-    const float hn = Elem<T>::to_f(static_cast<const T*>(ea.res)[size_t(m) * N + n]) + v;
+    const float hn = ea.res[size_t(m) * N + n] + v;
     const int b = m / ea.Kr;
     const size_t xrow = size_t(b) * ea.Lx + ea.idx[m];
-    T* o = static_cast<T*>(ea.out) + xrow * N + n;
-    const float x0 = Elem<T>::to_f(*o);
+    float* o = static_cast<float*>(ea.out) + xrow * N + n;
+    const float x0 = *o;
     const float delta = hn - x0;
-    *o = Elem<T>::from_f(x0 + delta);
+    *o = x0 + delta;
   }
 }
 
