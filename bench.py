@@ -304,7 +304,7 @@ def main():
     tokens = wl.B * wl.L * world
     value = tokens / (ms * 1e-3)
     roof, detail = roofline(trace, peaks, args.steps)
-    launches = sum(v["launches"] for k, v in trace.items() if k != "copy")
+    launches = sum(v["launches"] for v in trace.values())
     gs = {}
     for k in ("gather", "gemm_fc2_scatter"):
         if trace[k]["launches"]:

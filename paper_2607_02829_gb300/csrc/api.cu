@@ -170,6 +170,7 @@ cudaError_t gemm(const sr_handle* h, Epi epi, const void* A, const void* W, int 
 
 cudaError_t attention(const sr_handle* h, const void* qkv, void* out, int B, int T,
                       cudaStream_t s) {
+  if (h->dt == DType::BF16) return sr::launch_attention_tc(qkv, out, B, T, h->cfg.heads, h->fault(), s);
   return sr::launch_attention_simt(h->dt, qkv, out, B, T, h->cfg.heads, s);
 }
 

@@ -1,0 +1,322 @@
+// tcgen05 flash attention for head_dim 64, bf16 q/k/v, fp32 softmax statistics:
+// out[b, t, h*64 : h*64+64] = softmax(q k^T / 8) v over the T tokens of sample b
+// (the attention of the pre-LN block, Sec. 3.3 Eq. 11; within the sparse stage
+// T = K and the tokens are the routed ones, Eq. 8).  No mask; keys beyond T in
+// the last tile are excluded.
+//
+// One CTA owns 256 query rows of one (sample, head) as two 128-row tiles that
+// share every K/V tile, 320 threads:
+//   warp 0      TMA: the two Q tiles once, then K_j / V_j (128 keys x 64) into a
+//               3-stage ring (3-D tensor map over [B, T, 3D], zero fill past T);
+//   warp 1      tcgen05.mma: S^t = Q^t K_j^T (128 x 128, fp32 in TMEM) and
+//               O^t += P^t V_j (128 x 64, accumulated in TMEM), t = 0, 1;
+//   warps 2-5   softmax of tile 0, warps 6-9 softmax of tile 1: one query row
+//               per thread.  Each reads its S row from TMEM, updates the
+//               running max and sum, writes P = 2^(s*c - m*c) as bf16 into a
+//               128B-swizzled shared tile (the A operand of the P V MMA).
+// The running max is only raised when it grows by more than 2^8 (in the exp2
+// domain); then the thread rescales its O row in TMEM first.  P, O and the sum
+// always use the same max, so the result is exact up to rounding.
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc_ptx.cuh"
+
+namespace sr {
+namespace {
+
+using namespace tc;
+
+constexpr int kDh = 64;
+constexpr int kQTile = 128, kQTiles = 2, kBQ = kQTile * kQTiles;
+constexpr int kKV = 128;
+constexpr int kStages = 3;
+constexpr int kThreads = 320;
+constexpr int kTileBytes = kQTile * kDh * 2;                  // 16 KB: 128 rows x 128 B
+constexpr int kPBytes = kQTile * kKV * 2;                     // 32 KB: two 64-key atoms
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColS = 0;      // S^t at columns [128 t, 128 t + 128)
+constexpr uint32_t kColO = 256;    // O^t at columns [256 + 64 t, 256 + 64 t + 64)
+// raise the running max only when it grows by more than 8 in the exp2 domain
+constexpr float kRescaleLog2 = 8.0f;
+
+struct AttSmem {
+  uint64_t q_full, kv_full[kStages], kv_empty[kStages];
+  uint64_t s_full[kQTiles], p_full[kQTiles], pv_done[kQTiles], drain;
+  uint32_t tmem_base;
+  int abort;
+};
+
+constexpr size_t kSmemBytes = 1024 /*align*/ + size_t(kQTiles) * kTileBytes +
+                              size_t(kStages) * 2 * kTileBytes + size_t(kQTiles) * kPBytes + 256;
+
+__global__ void __launch_bounds__(kThreads, 1)
+attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ out, int T,
+                    int heads, unsigned int* fault) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* base = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  unsigned char* sQ = base;                                          // 2 x 16 KB
+  unsigned char* sKV = sQ + kQTiles * kTileBytes;                    // stages x (K 16 KB, V 16 KB)
+  unsigned char* sP = sKV + kStages * 2 * kTileBytes;                // 2 x 32 KB
+  AttSmem* sm = reinterpret_cast<AttSmem*>(sP + kQTiles * kPBytes);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qblocks = (T + kBQ - 1) / kBQ;
+  const int bh = blockIdx.x / qblocks;
+  const int qb = blockIdx.x % qblocks;
+  const int b = bh / heads, h = bh % heads;
+  const int D = heads * kDh;
+  const int q0 = qb * kBQ;
+  const int nkv = (T + kKV - 1) / kKV;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&sm->q_full, 1);
+    for (int s = 0; s < kStages; ++s) { mbar_init(&sm->kv_full[s], 1); mbar_init(&sm->kv_empty[s], 1); }
+    for (int t = 0; t < kQTiles; ++t) {
+      mbar_init(&sm->s_full[t], 1);
+      mbar_init(&sm->p_full[t], kQTile);
+      mbar_init(&sm->pv_done[t], 1);
+    }
+    mbar_init(&sm->drain, 1);
+    sm->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) prefetch_tmap(&tm);
+  if (warp == 1) tmem_alloc(&sm->tmem_base, kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm->tmem_base;
+  volatile int* abort = &sm->abort;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------- TMA loads
+    if (lane == 0) {
+      mbar_arrive_expect_tx(&sm->q_full, kQTiles * kTileBytes);
+      for (int t = 0; t < kQTiles; ++t)
+        tma_load_3d(&tm, sQ + t * kTileBytes, &sm->q_full, h * kDh, q0 + t * kQTile, b);
+      int stage = 0;
+      uint32_t phase = 0, issued = 0, issued_phase = 0;
+      for (int j = 0; j < nkv; ++j) {
+        if (!mbar_wait(&sm->kv_empty[stage], phase ^ 1, abort, fault)) break;
+        unsigned char* kt = sKV + size_t(stage) * 2 * kTileBytes;
+        mbar_arrive_expect_tx(&sm->kv_full[stage], 2 * kTileBytes);
+        tma_load_3d(&tm, kt, &sm->kv_full[stage], D + h * kDh, j * kKV, b);
+        tma_load_3d(&tm, kt + kTileBytes, &sm->kv_full[stage], 2 * D + h * kDh, j * kKV, b);
+        issued |= 1u << stage;
+        issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+        if (++stage == kStages) { stage = 0; phase ^= 1; }
+      }
+      // every issued load lands before the CTA may exit
+      int no_abort = 0;
+      mbar_wait(&sm->q_full, 0, &no_abort, fault);
+      for (int s = 0; s < kStages; ++s)
+        if (issued & (1u << s)) mbar_wait(&sm->kv_full[s], (issued_phase >> s) & 1u, &no_abort, fault);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------- MMA issue
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16(kQTile, kKV);                 // K-major A, B
+      constexpr uint32_t idesc_o = idesc_bf16(kQTile, kDh, false, true);   // V is MN-major
+      bool ok = mbar_wait(&sm->q_full, 0, abort, fault);
+      int stage = 0;
+      uint32_t phase = 0;
+      auto issue_s = [&](int t, int st) {
+        const uint32_t qa = smem_u32(sQ + t * kTileBytes);
+        const uint32_t ka = smem_u32(sKV + size_t(st) * 2 * kTileBytes);
+#pragma unroll
+        for (int k = 0; k < kDh / 16; ++k)
+          mma_bf16(tmem + kColS + uint32_t(t * kKV), sw128_desc(qa + 32 * k),
+                   sw128_desc(ka + 32 * k), idesc_s, k > 0 ? 1u : 0u);
+        mma_commit(&sm->s_full[t]);
+      };
+      if (ok) ok = mbar_wait(&sm->kv_full[0], 0, abort, fault);
+      if (ok) { issue_s(0, 0); issue_s(1, 0); }
+      for (int j = 0; j < nkv && ok; ++j) {
+        const int next = stage + 1 == kStages ? 0 : stage + 1;
+        const uint32_t next_phase = stage + 1 == kStages ? phase ^ 1 : phase;
+        for (int t = 0; t < kQTiles && ok; ++t) {
+          if (!(ok = mbar_wait(&sm->p_full[t], j & 1, abort, fault))) break;
+          tc_fence_after();
+          const uint32_t pa = smem_u32(sP + t * kPBytes);
+          const uint32_t va = smem_u32(sKV + size_t(stage) * 2 * kTileBytes + kTileBytes);
+#pragma unroll
+          for (int k = 0; k < kKV / 16; ++k)
+            mma_bf16(tmem + kColO + uint32_t(t * kDh),
+                     sw128_desc(pa + (k >> 2) * (kQTile * 128) + (k & 3) * 32),
+                     sw128_desc_mn(va + k * 2048), idesc_o, (j | k) != 0 ? 1u : 0u);
+          mma_commit(&sm->pv_done[t]);
+          if (j + 1 < nkv) {
+            if (t == 0 && !(ok = mbar_wait(&sm->kv_full[next], next_phase, abort, fault))) break;
+            issue_s(t, next);
+          }
+        }
+        mma_commit(&sm->kv_empty[stage]);
+        stage = next;
+        phase = next_phase;
+      }
+      int no_abort = 0;
+      mma_commit(&sm->drain);
+      mbar_wait(&sm->drain, 0, &no_abort, fault);
+    }
+  } else {
+    // ------------------------------------------------------------- softmax
+    const int t = (warp - 2) >> 2;                 // query tile of this warpgroup
+    const int quarter = warp & 3;                  // TMEM lane quarter
+    const int r = quarter * 32 + lane;             // row within the tile
+    const uint32_t lane_off = uint32_t(quarter * 32) << 16;
+    const uint32_t tS = tmem + lane_off + kColS + uint32_t(t * kKV);
+    const uint32_t tO = tmem + lane_off + kColO + uint32_t(t * kDh);
+    unsigned char* prow = sP + t * kPBytes + r * 128;
+    const float c = 0.125f * 1.4426950408889634f;  // 1/sqrt(64) * log2(e)
+    const float thresh = kRescaleLog2 / c;         // the same threshold in score units
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkv; ++j) {
+      ok = __all_sync(0xffffffffu, mbar_wait(&sm->s_full[t], j & 1, abort, fault));
+      if (!ok) break;
+      tc_fence_after();
+      uint32_t s[kKV / 32][32];
+#pragma unroll
+      for (int cc = 0; cc < kKV / 32; ++cc) tmem_ld32(tS + uint32_t(cc * 32), s[cc]);
+      tmem_wait_ld();
+      const int valid = T - j * kKV;               // keys of this tile that exist
+      float tmax = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < kKV; ++i) {
+        float v = __uint_as_float(s[i / 32][i % 32]);
+        if (i >= valid) v = -INFINITY;
+        s[i / 32][i % 32] = __float_as_uint(v);
+        tmax = fmaxf(tmax, v);
+      }
+      float alpha = 1.f;
+      bool rescale = false;
+      if (j == 0) {
+        m_run = tmax;
+      } else if (tmax > m_run + thresh) {
+        alpha = ex2((m_run - tmax) * c);
+        m_run = tmax;
+        l_run *= alpha;
+        rescale = true;
+      }
+      // the previous P V has finished reading P and accumulating into O
+      if (j > 0) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (j - 1) & 1, abort, fault));
+        if (!ok) break;
+        tc_fence_after();
+      }
+      if (__any_sync(0xffffffffu, rescale)) {
+        uint32_t o[32];
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          tmem_ld32(tO + uint32_t(half * 32), o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+          tmem_st32(tO + uint32_t(half * 32), o);
+        }
+        tmem_wait_st();
+      }
+      // P = 2^(s c - m c) as bf16 into the 128B-swizzled K-major tile: 16-byte
+      // chunk cc of the row goes to atom cc / 8, slot (cc % 8) ^ (r % 8)
+      const float mc = m_run * c;
+      float lsum = 0.f;
+#pragma unroll
+      for (int cc = 0; cc < kKV / 8; ++cc) {
+        uint32_t w[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int i0 = 8 * cc + 2 * q;
+          const float p0 = ex2(fmaf(__uint_as_float(s[i0 / 32][i0 % 32]), c, -mc));
+          const float p1 = ex2(fmaf(__uint_as_float(s[(i0 + 1) / 32][(i0 + 1) % 32]), c, -mc));
+          lsum += p0 + p1;
+          w[q] = pack_bf16x2(p0, p1);
+        }
+        const int atom = cc >> 3, slot = (cc & 7) ^ (r & 7);
+        *reinterpret_cast<uint4*>(prow + atom * (kQTile * 128) + slot * 16) =
+            make_uint4(w[0], w[1], w[2], w[3]);
+      }
+      l_run += lsum;
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(&sm->p_full[t]);
+    }
+    // epilogue: O / l for the rows that exist
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (nkv - 1) & 1, abort, fault));
+    if (ok) {
+      tc_fence_after();
+      uint32_t o[2][32];
+      tmem_ld32(tO, o[0]);
+      tmem_ld32(tO + 32, o[1]);
+      tmem_wait_ld();
+      const int row = q0 + t * kQTile + r;
+      if (row < T) {
+        const float inv = 1.f / l_run;
+        uint4* dst = reinterpret_cast<uint4*>(out + (size_t(b) * T + row) * D + h * kDh);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const uint32_t* q = &o[i / 4][(i % 4) * 8];
+          dst[i] = make_uint4(pack_bf16x2(__uint_as_float(q[0]) * inv, __uint_as_float(q[1]) * inv),
+                              pack_bf16x2(__uint_as_float(q[2]) * inv, __uint_as_float(q[3]) * inv),
+                              pack_bf16x2(__uint_as_float(q[4]) * inv, __uint_as_float(q[5]) * inv),
+                              pack_bf16x2(__uint_as_float(q[6]) * inv, __uint_as_float(q[7]) * inv));
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+cudaError_t get_encoder() {
+  if (g_encode) return cudaSuccess;
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                   cudaEnableDefault, &q);
+  if (e != cudaSuccess) return e;
+  if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+  g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_attention_tc(const void* qkv, void* out, int B, int T, int heads,
+                                unsigned int* fault, cudaStream_t s) {
+  cudaError_t e = get_encoder();
+  if (e != cudaSuccess) return e;
+  const uint64_t D3 = uint64_t(3) * heads * kDh;
+  // [B, T, 3D] bf16, box: 64 columns x 128 tokens x 1 sample
+  CUtensorMap tm;
+  cuuint64_t dims[3] = {D3, uint64_t(T), uint64_t(B)};
+  cuuint64_t strides[2] = {D3 * 2, D3 * 2 * uint64_t(T)};
+  cuuint32_t box[3] = {kDh, kKV, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(&tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(qkv), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  static bool attr_set = false;
+  if (!attr_set) {
+    e = cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             int(kSmemBytes));
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const int grid = B * heads * ((T + kBQ - 1) / kBQ);
+  attention_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(tm, static_cast<bf16*>(out), T, heads,
+                                                         fault);
+  return cudaGetLastError();
+}
+
+}  // namespace sr

@@ -198,7 +198,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       const int mt = t % m_tiles, nt = t / m_tiles;
       const int acc = it & 1;
       const uint32_t aphase = (it >> 1) & 1;
-      if (!mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault)) break;
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault))) break;
       tc_fence_after();
       const int m = mt * BM + row;
       const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);

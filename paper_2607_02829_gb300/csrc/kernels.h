@@ -68,7 +68,10 @@ cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* Bw, int M, int N,
 
 // ---- attention core: per (sample, head) softmax(q k^T / sqrt(64)) v ------
 // qkv [B*T, 3D] (q | k | v, head h at columns 64h..64h+63 of each); out [B*T, D].
+// CUDA-core version (fp32 storage) and tcgen05 version (bf16 storage).
 cudaError_t launch_attention_simt(DType dt, const void* qkv, void* out, int B, int T, int heads,
                                   cudaStream_t s);
+cudaError_t launch_attention_tc(const void* qkv, void* out, int B, int T, int heads,
+                                unsigned int* fault, cudaStream_t s);
 
 }  // namespace sr
