@@ -175,6 +175,32 @@ sr_status sr_trace_read(sr_handle* h, sr_trace_entry* out, int reset);
 /* Releases the handle (not the workspace, which the caller owns).  NULL is a no-op. */
 sr_status sr_destroy(sr_handle* h);
 
+/* ---- allocation-free variant of the top-K L2-norm selector ---------------
+ * The paper has no counterpart of this call; it exists for callers that cannot
+ * allocate device memory: a plugin running inside a host framework that owns
+ * the GPU's memory pool and hands it no workspace, or a latency-critical path
+ * on which cudaMalloc's implicit device synchronisation is not acceptable.
+ * It computes exactly what sr_select computes with SR_SEL_TOPK_L2 for the same
+ * x, B, L, D, dtype and keep_ratio, but needs no handle and no workspace: its
+ * per-token score scratch is a static device array of 1,048,576 floats (4 MiB)
+ * compiled into this library, which every GPU that loads the library keeps
+ * until the process exits.
+ *  x        : [B, L, D] device, dtype storage (SR_F32 / SR_BF16), 16-byte aligned.
+ *  idx      : [B, K] int32 device output, each row strictly increasing.
+ *  K_out    : host int32, receives K = floor(L * keep_ratio) (may be NULL).
+ * Returns SR_ERR_UNSUPPORTED when B * L exceeds 1,048,576 (or L or D exceed
+ * what the selection kernels support), SR_ERR_INVALID_ARG for bad pointers,
+ * dtype or ratio, before any launch.  Calls no cudaMalloc, cudaFree or other
+ * allocating routine.  The first call on each device looks up the static
+ * array's device address (cudaGetSymbolAddress); make that first call before
+ * any stream capture.  All calls share the one array and it keeps the last
+ * call's scores; each call overwrites every score it reads, so nothing has to
+ * start at zero, but calls whose work overlaps on the GPU (other streams, or
+ * other host threads on the same device) race on it and must be serialised
+ * by the caller. */
+sr_status sr_select_topk_l2_static(const void* x, int32_t B, int32_t L, int32_t D, int32_t dtype,
+                                   float keep_ratio, int32_t* idx, int32_t* K_out, void* stream);
+
 /* Static description of a status code. */
 const char* sr_status_string(sr_status s);
 

@@ -81,6 +81,9 @@ def lib() -> ctypes.CDLL:
         L.sr_trace_read.restype = st
         L.sr_device_fault.argtypes = [vp, ctypes.POINTER(ctypes.c_uint32), ctypes.c_int, vp]
         L.sr_device_fault.restype = st
+        L.sr_select_topk_l2_static.argtypes = [vp, i32, i32, i32, i32, ctypes.c_float, vp,
+                                               ctypes.POINTER(i32), vp]
+        L.sr_select_topk_l2_static.restype = st
         L.sr_status_string.argtypes = [st]; L.sr_status_string.restype = ctypes.c_char_p
         L.sr_last_error_message.argtypes = []; L.sr_last_error_message.restype = ctypes.c_char_p
         _lib = L
@@ -150,6 +153,14 @@ def sr_device_fault(handle: int, clear: bool, stream: int) -> int:
     _check(lib().sr_device_fault(handle, ctypes.byref(f), int(bool(clear)), stream),
            "sr_device_fault")
     return f.value
+
+
+def sr_select_topk_l2_static(x: int, B: int, L: int, D: int, dtype: int, keep_ratio: float,
+                             idx: int, stream: int) -> int:
+    K = ctypes.c_int32(0)
+    _check(lib().sr_select_topk_l2_static(x, B, L, D, dtype, keep_ratio, idx, ctypes.byref(K),
+                                          stream), "sr_select_topk_l2_static")
+    return K.value
 
 
 # ----------------------------------------------------- torch-side helpers

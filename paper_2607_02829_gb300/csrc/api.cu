@@ -15,6 +15,10 @@
 using sr::DType;
 using sr::Epi;
 
+namespace sr {
+void set_error_message(const std::string& msg);
+}  // namespace sr
+
 namespace {
 
 thread_local std::string g_last_msg;
@@ -37,6 +41,14 @@ sr_status cuda_fail(cudaError_t e, const char* where) {
 
 constexpr size_t kAlign = 256;
 size_t align_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
+
+}  // namespace
+
+// Records a message for sr_last_error_message() (used by entry points defined
+// in other translation units).
+void sr::set_error_message(const std::string& msg) { g_last_msg = msg; }
+
+namespace {
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
