@@ -9,7 +9,9 @@
 //   warp 0      TMA: the two Q tiles once, then K_j / V_j (128 keys x 64) into a
 //               3-stage ring (3-D tensor map over [B, T, 3D], zero fill past T);
 //   warp 1      tcgen05.mma: S^t = Q^t K_j^T (128 x 128, fp32 in TMEM) and
-//               O^t += P^t V_j (128 x 64, accumulated in TMEM), t = 0, 1;
+//               O^t += P^t V_j (128 x 64, accumulated in TMEM), t = 0, 1; the
+//               next S^t is issued as soon as softmax t has read the current
+//               one, so it is ready when the softmax needs it;
 //   warps 2-5   softmax of tile 0, warps 6-9 softmax of tile 1: one query row
 //               per thread.  Each reads its S row from TMEM, updates the
 //               running max and sum, writes P = 2^(s*c - m*c) as bf16 into a
@@ -43,7 +45,7 @@ constexpr float kRescaleLog2 = 8.0f;
 
 struct AttSmem {
   uint64_t q_full, kv_full[kStages], kv_empty[kStages];
-  uint64_t s_full[kQTiles], p_full[kQTiles], pv_done[kQTiles], drain;
+  uint64_t s_full[kQTiles], s_free[kQTiles], p_full[kQTiles], pv_done[kQTiles], drain;
   uint32_t tmem_base;
   int abort;
 };
@@ -76,6 +78,7 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
     for (int s = 0; s < kStages; ++s) { mbar_init(&sm->kv_full[s], 1); mbar_init(&sm->kv_empty[s], 1); }
     for (int t = 0; t < kQTiles; ++t) {
       mbar_init(&sm->s_full[t], 1);
+      mbar_init(&sm->s_free[t], kQTile);
       mbar_init(&sm->p_full[t], kQTile);
       mbar_init(&sm->pv_done[t], 1);
     }
@@ -137,6 +140,16 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
       for (int j = 0; j < nkv && ok; ++j) {
         const int next = stage + 1 == kStages ? 0 : stage + 1;
         const uint32_t next_phase = stage + 1 == kStages ? phase ^ 1 : phase;
+        // S for the next key tile as soon as each softmax has read its S row
+        if (j + 1 < nkv) {
+          if (!(ok = mbar_wait(&sm->kv_full[next], next_phase, abort, fault))) break;
+          for (int t = 0; t < kQTiles && ok; ++t) {
+            if (!(ok = mbar_wait(&sm->s_free[t], j & 1, abort, fault))) break;
+            tc_fence_after();
+            issue_s(t, next);
+          }
+          if (!ok) break;
+        }
         for (int t = 0; t < kQTiles && ok; ++t) {
           if (!(ok = mbar_wait(&sm->p_full[t], j & 1, abort, fault))) break;
           tc_fence_after();
@@ -148,10 +161,6 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
                      sw128_desc(pa + (k >> 2) * (kQTile * 128) + (k & 3) * 32),
                      sw128_desc_mn(va + k * 2048), idesc_o, (j | k) != 0 ? 1u : 0u);
           mma_commit(&sm->pv_done[t]);
-          if (j + 1 < nkv) {
-            if (t == 0 && !(ok = mbar_wait(&sm->kv_full[next], next_phase, abort, fault))) break;
-            issue_s(t, next);
-          }
         }
         mma_commit(&sm->kv_empty[stage]);
         stage = next;
@@ -182,15 +191,21 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
 #pragma unroll
       for (int cc = 0; cc < kKV / 32; ++cc) tmem_ld32(tS + uint32_t(cc * 32), s[cc]);
       tmem_wait_ld();
+      tc_fence_before();
+      mbar_arrive(&sm->s_free[t]);                 // S may now be overwritten
       const int valid = T - j * kKV;               // keys of this tile that exist
-      float tmax = -INFINITY;
+      if (valid < kKV) {
 #pragma unroll
-      for (int i = 0; i < kKV; ++i) {
-        float v = __uint_as_float(s[i / 32][i % 32]);
-        if (i >= valid) v = -INFINITY;
-        s[i / 32][i % 32] = __float_as_uint(v);
-        tmax = fmaxf(tmax, v);
+        for (int i = 0; i < kKV; ++i)
+          if (i >= valid) s[i / 32][i % 32] = __float_as_uint(-INFINITY);
       }
+      float pm[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) pm[k] = __uint_as_float(s[0][k]);
+#pragma unroll
+      for (int i = 8; i < kKV; ++i) pm[i % 8] = fmaxf(pm[i % 8], __uint_as_float(s[i / 32][i % 32]));
+      const float tmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
       float alpha = 1.f;
       bool rescale = false;
       if (j == 0) {
@@ -207,6 +222,27 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
         if (!ok) break;
         tc_fence_after();
       }
+      // P = 2^(s c - m c) as bf16 into the 128B-swizzled K-major tile: 16-byte
+      // chunk cc of the row goes to atom cc / 8, slot (cc % 8) ^ (r % 8)
+      const float mc = m_run * c;
+      float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int cc = 0; cc < kKV / 8; ++cc) {
+        uint32_t w[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int i0 = 8 * cc + 2 * q;
+          const float p0 = ex2(fmaf(__uint_as_float(s[i0 / 32][i0 % 32]), c, -mc));
+          const float p1 = ex2(fmaf(__uint_as_float(s[(i0 + 1) / 32][(i0 + 1) % 32]), c, -mc));
+          ls[q] += p0 + p1;
+          w[q] = pack_bf16x2(p0, p1);
+        }
+        const int atom = cc >> 3, slot = (cc & 7) ^ (r & 7);
+        *reinterpret_cast<uint4*>(prow + atom * (kQTile * 128) + slot * 16) =
+            make_uint4(w[0], w[1], w[2], w[3]);
+      }
+      l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+      // O (all previous P V products, complete) follows a raised max
       if (__any_sync(0xffffffffu, rescale)) {
         uint32_t o[32];
 #pragma unroll
@@ -219,26 +255,6 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
         }
         tmem_wait_st();
       }
-      // P = 2^(s c - m c) as bf16 into the 128B-swizzled K-major tile: 16-byte
-      // chunk cc of the row goes to atom cc / 8, slot (cc % 8) ^ (r % 8)
-      const float mc = m_run * c;
-      float lsum = 0.f;
-#pragma unroll
-      for (int cc = 0; cc < kKV / 8; ++cc) {
-        uint32_t w[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int i0 = 8 * cc + 2 * q;
-          const float p0 = ex2(fmaf(__uint_as_float(s[i0 / 32][i0 % 32]), c, -mc));
-          const float p1 = ex2(fmaf(__uint_as_float(s[(i0 + 1) / 32][(i0 + 1) % 32]), c, -mc));
-          lsum += p0 + p1;
-          w[q] = pack_bf16x2(p0, p1);
-        }
-        const int atom = cc >> 3, slot = (cc & 7) ^ (r & 7);
-        *reinterpret_cast<uint4*>(prow + atom * (kQTile * 128) + slot * 16) =
-            make_uint4(w[0], w[1], w[2], w[3]);
-      }
-      l_run += lsum;
       fence_proxy_async_smem();
       tc_fence_before();
       mbar_arrive(&sm->p_full[t]);
