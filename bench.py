@@ -40,14 +40,19 @@ def _peaks():
                 "source": "fallback"}
 
 
-def _workload(name):
+def _workload(name, split=None):
     from paper_2607_02829_gb300 import synth
-    if name in synth.WORKLOADS:
-        return synth.WORKLOADS[name]
-    for wl in synth.sweep_workloads():
-        if wl.name == name:
-            return wl
-    raise SystemExit(f"unknown workload {name}")
+    wl = synth.WORKLOADS.get(name)
+    if wl is None:
+        for w in synth.sweep_workloads():
+            if w.name == name:
+                wl = w
+    if wl is None:
+        raise SystemExit(f"unknown workload {name}")
+    if split:
+        n1, n2, n3 = (int(v) for v in split.split(","))
+        wl = wl.with_(name=f"{wl.name}_split{n1}-{n2}-{n3}", n1=n1, n2=n2, n3=n3)
+    return wl
 
 
 def _describe(wl, K):
@@ -118,7 +123,7 @@ def run_ours(args, rank, world, local_rank):
 
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    wl = _workload(args.workload)
+    wl = _workload(args.workload, args.split)
     K = b.sr_keep_count(wl.L, wl.keep_ratio)
     cfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, wl.n1, wl.n2, wl.n3, dtype=wl.dtype,
                         selector=wl.selector)
@@ -276,6 +281,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--split", default=None,
+                    help="override the block split n1,n2,n3 (kernel studies and profiling)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -340,7 +347,7 @@ def run_reference(args, rank, world):
     """The oracle as the reference arm, on the host cores, rank 0 only."""
     if rank != 0:
         return
-    wl = _workload(args.workload)
+    wl = _workload(args.workload, args.split)
     from oracle import reslim as o
     K = o.keep_count(wl.L, wl.keep_ratio)
     vals = []

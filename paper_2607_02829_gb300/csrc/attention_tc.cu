@@ -5,17 +5,20 @@
 // the last tile are excluded.
 //
 // One CTA owns 256 query rows of one (sample, head) as two 128-row tiles that
-// share every K/V tile, 320 threads:
-//   warp 0      TMA: the two Q tiles once, then K_j / V_j (128 keys x 64) into a
-//               3-stage ring (3-D tensor map over [B, T, 3D], zero fill past T);
-//   warp 1      tcgen05.mma: S^t = Q^t K_j^T (128 x 128, fp32 in TMEM) and
-//               O^t += P^t V_j (128 x 64, accumulated in TMEM), t = 0, 1; the
-//               next S^t is issued as soon as softmax t has read the current
-//               one, so it is ready when the softmax needs it;
-//   warps 2-5   softmax of tile 0, warps 6-9 softmax of tile 1: one query row
+// share every K/V tile, 384 threads:
+//   warps 0, 3  TMA: the two Q tiles once, then K_j (warp 0) and V_j (warp 3),
+//               128 keys x 64, into two 2-stage rings (3-D tensor map over
+//               [B, T, 3D], zero fill past T); a K stage frees as soon as both
+//               tiles' S MMAs that read it finish, a V stage when the P V MMAs do;
+//   warps 1, 2  tcgen05.mma for tile 0 and tile 1, each thread in its own order:
+//               S^t = Q^t K_j^T (128 x 128, fp32 in TMEM), O^t += P^t V_j
+//               (128 x 64, accumulated in TMEM); the next S^t is issued as soon
+//               as softmax t has read the current one;
+//   warps 4-7   softmax of tile 0, warps 8-11 softmax of tile 1: one query row
 //               per thread.  Each reads its S row from TMEM, updates the
-//               running max and sum, writes P = 2^(s*c - m*c) as bf16 into a
-//               128B-swizzled shared tile (the A operand of the P V MMA).
+//               running max and sum, writes P = 2^(s*c - m*c) as bf16 into one
+//               of two 128B-swizzled shared tiles (the A operand of the P V
+//               MMA), so P of the next key tile never waits for this P V.
 // The running max is only raised when it grows by more than 2^8 (in the exp2
 // domain); then the thread rescales its O row in TMEM first.  P, O and the sum
 // always use the same max, so the result is exact up to rounding.
@@ -33,8 +36,8 @@ using namespace tc;
 constexpr int kDh = 64;
 constexpr int kQTile = 128, kQTiles = 2, kBQ = kQTile * kQTiles;
 constexpr int kKV = 128;
-constexpr int kStages = 3;
-constexpr int kThreads = 320;
+constexpr int kStages = 2;                                    // K ring and V ring
+constexpr int kThreads = 384;
 constexpr int kTileBytes = kQTile * kDh * 2;                  // 16 KB: 128 rows x 128 B
 constexpr int kPBytes = kQTile * kKV * 2;                     // 32 KB: two 64-key atoms
 constexpr uint32_t kTmemCols = 512;
@@ -44,14 +47,41 @@ constexpr uint32_t kColO = 256;    // O^t at columns [256 + 64 t, 256 + 64 t + 6
 constexpr float kRescaleLog2 = 8.0f;
 
 struct AttSmem {
-  uint64_t q_full, kv_full[kStages], kv_empty[kStages];
-  uint64_t s_full[kQTiles], s_free[kQTiles], p_full[kQTiles], pv_done[kQTiles], drain;
+  uint64_t q_full;
+  uint64_t k_full[kStages], k_empty[kStages], v_full[kStages], v_empty[kStages];
+  uint64_t s_full[kQTiles], s_free[kQTiles], p_full[kQTiles][2], pv_done[kQTiles][2];
+  uint64_t drain[kQTiles];
   uint32_t tmem_base;
   int abort;
 };
 
 constexpr size_t kSmemBytes = 1024 /*align*/ + size_t(kQTiles) * kTileBytes +
-                              size_t(kStages) * 2 * kTileBytes + size_t(kQTiles) * kPBytes + 256;
+                              size_t(kStages) * 2 * kTileBytes + size_t(kQTiles) * 2 * kPBytes + 256;
+
+// packed fp32 pairs (the f32x2 instructions of sm_100+)
+__device__ __forceinline__ uint64_t pk2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void up2(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
 
 __global__ void __launch_bounds__(kThreads, 1)
 attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ out, int T,
@@ -59,10 +89,11 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  unsigned char* sQ = base;                                          // 2 x 16 KB
-  unsigned char* sKV = sQ + kQTiles * kTileBytes;                    // stages x (K 16 KB, V 16 KB)
-  unsigned char* sP = sKV + kStages * 2 * kTileBytes;                // 2 x 32 KB
-  AttSmem* sm = reinterpret_cast<AttSmem*>(sP + kQTiles * kPBytes);
+  unsigned char* sQ = base;                                  // 2 x 16 KB
+  unsigned char* sK = sQ + kQTiles * kTileBytes;             // 2 stages x 16 KB
+  unsigned char* sV = sK + kStages * kTileBytes;             // 2 stages x 16 KB
+  unsigned char* sP = sV + kStages * kTileBytes;             // [tile][buffer] x 32 KB
+  AttSmem* sm = reinterpret_cast<AttSmem*>(sP + kQTiles * 2 * kPBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qblocks = (T + kBQ - 1) / kBQ;
@@ -75,14 +106,20 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
 
   if (threadIdx.x == 0) {
     mbar_init(&sm->q_full, 1);
-    for (int s = 0; s < kStages; ++s) { mbar_init(&sm->kv_full[s], 1); mbar_init(&sm->kv_empty[s], 1); }
+    for (int s = 0; s < kStages; ++s) {
+      // a stage is released by both MMA threads
+      mbar_init(&sm->k_full[s], 1); mbar_init(&sm->k_empty[s], kQTiles);
+      mbar_init(&sm->v_full[s], 1); mbar_init(&sm->v_empty[s], kQTiles);
+    }
     for (int t = 0; t < kQTiles; ++t) {
       mbar_init(&sm->s_full[t], 1);
       mbar_init(&sm->s_free[t], kQTile);
-      mbar_init(&sm->p_full[t], kQTile);
-      mbar_init(&sm->pv_done[t], 1);
+      for (int bf = 0; bf < 2; ++bf) {
+        mbar_init(&sm->p_full[t][bf], kQTile);
+        mbar_init(&sm->pv_done[t][bf], 1);
+      }
+      mbar_init(&sm->drain[t], 1);
     }
-    mbar_init(&sm->drain, 1);
     sm->abort = 0;
     fence_mbar_init();
   }
@@ -94,93 +131,99 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
   const uint32_t tmem = sm->tmem_base;
   volatile int* abort = &sm->abort;
 
-  if (warp == 0) {
+  if (warp == 0 || warp == 3) {
     // ------------------------------------------------------------- TMA loads
+    // warp 0: the Q tiles, then K_j; warp 3: V_j
     if (lane == 0) {
-      mbar_arrive_expect_tx(&sm->q_full, kQTiles * kTileBytes);
-      for (int t = 0; t < kQTiles; ++t)
-        tma_load_3d(&tm, sQ + t * kTileBytes, &sm->q_full, h * kDh, q0 + t * kQTile, b);
-      int stage = 0;
-      uint32_t phase = 0, issued = 0, issued_phase = 0;
+      const bool is_k = warp == 0;
+      if (is_k) {
+        mbar_arrive_expect_tx(&sm->q_full, kQTiles * kTileBytes);
+        for (int t = 0; t < kQTiles; ++t)
+          tma_load_3d(&tm, sQ + t * kTileBytes, &sm->q_full, h * kDh, q0 + t * kQTile, b);
+      }
+      uint64_t* full = is_k ? sm->k_full : sm->v_full;
+      uint64_t* empty = is_k ? sm->k_empty : sm->v_empty;
+      unsigned char* ring = is_k ? sK : sV;
+      const int col = (is_k ? D : 2 * D) + h * kDh;
+      uint32_t issued = 0, par = 0;   // stages holding a load; parity of its phase
       for (int j = 0; j < nkv; ++j) {
-        if (!mbar_wait(&sm->kv_empty[stage], phase ^ 1, abort, fault)) break;
-        unsigned char* kt = sKV + size_t(stage) * 2 * kTileBytes;
-        mbar_arrive_expect_tx(&sm->kv_full[stage], 2 * kTileBytes);
-        tma_load_3d(&tm, kt, &sm->kv_full[stage], D + h * kDh, j * kKV, b);
-        tma_load_3d(&tm, kt + kTileBytes, &sm->kv_full[stage], 2 * D + h * kDh, j * kKV, b);
-        issued |= 1u << stage;
-        issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-        if (++stage == kStages) { stage = 0; phase ^= 1; }
+        const int st = j & 1;
+        const uint32_t ph = (j >> 1) & 1;
+        // the stage is free once both tiles' MMAs of key tile j - 2 have read it
+        if (!mbar_wait(&empty[st], ph ^ 1, abort, fault)) break;
+        mbar_arrive_expect_tx(&full[st], kTileBytes);
+        tma_load_3d(&tm, ring + st * kTileBytes, &full[st], col, j * kKV, b);
+        issued |= 1u << st;
+        par = (par & ~(1u << st)) | (ph << st);
       }
       // every issued load lands before the CTA may exit
       int no_abort = 0;
-      mbar_wait(&sm->q_full, 0, &no_abort, fault);
+      if (is_k) mbar_wait(&sm->q_full, 0, &no_abort, fault);
       for (int s = 0; s < kStages; ++s)
-        if (issued & (1u << s)) mbar_wait(&sm->kv_full[s], (issued_phase >> s) & 1u, &no_abort, fault);
+        if (issued & (1u << s)) mbar_wait(&full[s], (par >> s) & 1u, &no_abort, fault);
     }
-  } else if (warp == 1) {
+  } else if (warp == 1 || warp == 2) {
     // ------------------------------------------------------------- MMA issue
+    // warp 1 issues tile 0's MMAs, warp 2 tile 1's, each in its own order
     if (lane == 0) {
+      const int t = warp - 1;
       constexpr uint32_t idesc_s = idesc_bf16(kQTile, kKV);                 // K-major A, B
       constexpr uint32_t idesc_o = idesc_bf16(kQTile, kDh, false, true);   // V is MN-major
-      bool ok = mbar_wait(&sm->q_full, 0, abort, fault);
-      int stage = 0;
-      uint32_t phase = 0;
-      auto issue_s = [&](int t, int st) {
-        const uint32_t qa = smem_u32(sQ + t * kTileBytes);
-        const uint32_t ka = smem_u32(sKV + size_t(st) * 2 * kTileBytes);
+      const uint32_t dS = tmem + kColS + uint32_t(t * kKV);
+      const uint32_t dO = tmem + kColO + uint32_t(t * kDh);
+      const uint32_t qa = smem_u32(sQ + t * kTileBytes);
+      auto issue_s = [&](int st) {
+        const uint32_t ka = smem_u32(sK + st * kTileBytes);
 #pragma unroll
         for (int k = 0; k < kDh / 16; ++k)
-          mma_bf16(tmem + kColS + uint32_t(t * kKV), sw128_desc(qa + 32 * k),
-                   sw128_desc(ka + 32 * k), idesc_s, k > 0 ? 1u : 0u);
+          mma_bf16(dS, sw128_desc(qa + 32 * k), sw128_desc(ka + 32 * k), idesc_s, k > 0 ? 1u : 0u);
         mma_commit(&sm->s_full[t]);
+        mma_commit(&sm->k_empty[st]);
       };
-      if (ok) ok = mbar_wait(&sm->kv_full[0], 0, abort, fault);
-      if (ok) { issue_s(0, 0); issue_s(1, 0); }
+      bool ok = mbar_wait(&sm->q_full, 0, abort, fault);
+      if (ok) ok = mbar_wait(&sm->k_full[0], 0, abort, fault);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0);
+      }
       for (int j = 0; j < nkv && ok; ++j) {
-        const int next = stage + 1 == kStages ? 0 : stage + 1;
-        const uint32_t next_phase = stage + 1 == kStages ? phase ^ 1 : phase;
-        // S for the next key tile as soon as each softmax has read its S row
+        // S for the next key tile as soon as the softmax has read this one
         if (j + 1 < nkv) {
-          if (!(ok = mbar_wait(&sm->kv_full[next], next_phase, abort, fault))) break;
-          for (int t = 0; t < kQTiles && ok; ++t) {
-            if (!(ok = mbar_wait(&sm->s_free[t], j & 1, abort, fault))) break;
-            tc_fence_after();
-            issue_s(t, next);
-          }
-          if (!ok) break;
-        }
-        for (int t = 0; t < kQTiles && ok; ++t) {
-          if (!(ok = mbar_wait(&sm->p_full[t], j & 1, abort, fault))) break;
+          const int st = (j + 1) & 1;
+          if (!(ok = mbar_wait(&sm->k_full[st], ((j + 1) >> 1) & 1, abort, fault))) break;
+          if (!(ok = mbar_wait(&sm->s_free[t], j & 1, abort, fault))) break;
           tc_fence_after();
-          const uint32_t pa = smem_u32(sP + t * kPBytes);
-          const uint32_t va = smem_u32(sKV + size_t(stage) * 2 * kTileBytes + kTileBytes);
-#pragma unroll
-          for (int k = 0; k < kKV / 16; ++k)
-            mma_bf16(tmem + kColO + uint32_t(t * kDh),
-                     sw128_desc(pa + (k >> 2) * (kQTile * 128) + (k & 3) * 32),
-                     sw128_desc_mn(va + k * 2048), idesc_o, (j | k) != 0 ? 1u : 0u);
-          mma_commit(&sm->pv_done[t]);
+          issue_s(st);
         }
-        mma_commit(&sm->kv_empty[stage]);
-        stage = next;
-        phase = next_phase;
+        // O^t += P^t_j V_j
+        const int vs = j & 1;
+        if (!(ok = mbar_wait(&sm->v_full[vs], (j >> 1) & 1, abort, fault))) break;
+        if (!(ok = mbar_wait(&sm->p_full[t][j & 1], (j >> 1) & 1, abort, fault))) break;
+        tc_fence_after();
+        const uint32_t pa = smem_u32(sP + (t * 2 + (j & 1)) * kPBytes);
+        const uint32_t va = smem_u32(sV + vs * kTileBytes);
+#pragma unroll
+        for (int k = 0; k < kKV / 16; ++k)
+          mma_bf16(dO, sw128_desc(pa + (k >> 2) * (kQTile * 128) + (k & 3) * 32),
+                   sw128_desc_mn(va + k * 2048), idesc_o, (j | k) != 0 ? 1u : 0u);
+        mma_commit(&sm->pv_done[t][j & 1]);
+        mma_commit(&sm->v_empty[vs]);
       }
       int no_abort = 0;
-      mma_commit(&sm->drain);
-      mbar_wait(&sm->drain, 0, &no_abort, fault);
+      mma_commit(&sm->drain[t]);
+      mbar_wait(&sm->drain[t], 0, &no_abort, fault);
     }
   } else {
     // ------------------------------------------------------------- softmax
-    const int t = (warp - 2) >> 2;                 // query tile of this warpgroup
+    const int t = (warp - 4) >> 2;                 // query tile of this warpgroup
     const int quarter = warp & 3;                  // TMEM lane quarter
     const int r = quarter * 32 + lane;             // row within the tile
     const uint32_t lane_off = uint32_t(quarter * 32) << 16;
     const uint32_t tS = tmem + lane_off + kColS + uint32_t(t * kKV);
     const uint32_t tO = tmem + lane_off + kColO + uint32_t(t * kDh);
-    unsigned char* prow = sP + t * kPBytes + r * 128;
     const float c = 0.125f * 1.4426950408889634f;  // 1/sqrt(64) * log2(e)
     const float thresh = kRescaleLog2 / c;         // the same threshold in score units
+    const uint64_t c2 = pk2(c, c);
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int j = 0; j < nkv; ++j) {
@@ -199,13 +242,22 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
         for (int i = 0; i < kKV; ++i)
           if (i >= valid) s[i / 32][i % 32] = __float_as_uint(-INFINITY);
       }
+      // row max: eight chains of three-input maxima
       float pm[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) pm[k] = __uint_as_float(s[0][k]);
 #pragma unroll
-      for (int i = 8; i < kKV; ++i) pm[i % 8] = fmaxf(pm[i % 8], __uint_as_float(s[i / 32][i % 32]));
-      const float tmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+      for (int i = 8; i < kKV; i += 16) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int a = i + k, bb = i + 8 + k;
+          pm[k] = bb < kKV ? max3(pm[k], __uint_as_float(s[a / 32][a % 32]),
+                                  __uint_as_float(s[bb / 32][bb % 32]))
+                           : fmaxf(pm[k], __uint_as_float(s[a / 32][a % 32]));
+        }
+      }
+      const float tmax = max3(max3(pm[0], pm[1], pm[2]), max3(pm[3], pm[4], pm[5]),
+                              fmaxf(pm[6], pm[7]));
       float alpha = 1.f;
       bool rescale = false;
       if (j == 0) {
@@ -216,34 +268,49 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
         l_run *= alpha;
         rescale = true;
       }
-      // the previous P V has finished reading P and accumulating into O
-      if (j > 0) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (j - 1) & 1, abort, fault));
+      // P buffer j % 2 was last read by P V of tile j - 2
+      if (j >= 2) {
+        ok = __all_sync(0xffffffffu,
+                        mbar_wait(&sm->pv_done[t][j & 1], ((j >> 1) & 1) ^ 1, abort, fault));
         if (!ok) break;
-        tc_fence_after();
       }
       // P = 2^(s c - m c) as bf16 into the 128B-swizzled K-major tile: 16-byte
       // chunk cc of the row goes to atom cc / 8, slot (cc % 8) ^ (r % 8)
+      unsigned char* prow = sP + (t * 2 + (j & 1)) * kPBytes + r * 128;
       const float mc = m_run * c;
-      float ls[4] = {0.f, 0.f, 0.f, 0.f};
+      const uint64_t nmc2 = pk2(-mc, -mc);
+      uint64_t ls2[2] = {pk2(0.f, 0.f), pk2(0.f, 0.f)};
 #pragma unroll
       for (int cc = 0; cc < kKV / 8; ++cc) {
         uint32_t w[4];
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           const int i0 = 8 * cc + 2 * q;
-          const float p0 = ex2(fmaf(__uint_as_float(s[i0 / 32][i0 % 32]), c, -mc));
-          const float p1 = ex2(fmaf(__uint_as_float(s[(i0 + 1) / 32][(i0 + 1) % 32]), c, -mc));
-          ls[q] += p0 + p1;
+          const uint64_t arg = fma2(pk2(__uint_as_float(s[i0 / 32][i0 % 32]),
+                                        __uint_as_float(s[(i0 + 1) / 32][(i0 + 1) % 32])),
+                                    c2, nmc2);
+          float a0, a1;
+          up2(arg, a0, a1);
+          const float p0 = ex2(a0), p1 = ex2(a1);
+          ls2[q & 1] = add2(ls2[q & 1], pk2(p0, p1));
           w[q] = pack_bf16x2(p0, p1);
         }
         const int atom = cc >> 3, slot = (cc & 7) ^ (r & 7);
         *reinterpret_cast<uint4*>(prow + atom * (kQTile * 128) + slot * 16) =
             make_uint4(w[0], w[1], w[2], w[3]);
       }
-      l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-      // O (all previous P V products, complete) follows a raised max
+      {
+        float l0, l1, l2, l3;
+        up2(ls2[0], l0, l1);
+        up2(ls2[1], l2, l3);
+        l_run += (l0 + l1) + (l2 + l3);
+      }
+      // a raised max rescales O, which then holds every earlier P V product
       if (__any_sync(0xffffffffu, rescale)) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t][(j - 1) & 1],
+                                               ((j - 1) >> 1) & 1, abort, fault));
+        if (!ok) break;
+        tc_fence_after();
         uint32_t o[32];
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
@@ -257,10 +324,12 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
       }
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(&sm->p_full[t]);
+      mbar_arrive(&sm->p_full[t][j & 1]);
     }
-    // epilogue: O / l for the rows that exist
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (nkv - 1) & 1, abort, fault));
+    // epilogue: O / l for the rows that exist (the last P V implies all earlier ones)
+    if (ok)
+      ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t][(nkv - 1) & 1],
+                                             ((nkv - 1) >> 1) & 1, abort, fault));
     if (ok) {
       tc_fence_after();
       uint32_t o[2][32];
