@@ -2,14 +2,15 @@
 // the block's epilogues fused (bias; bias + GELU; bias + fp32 residual add; bias
 // + residual + the delta scatter of Eq. 9 for the last sparse block).
 //
-// Persistent, warp-specialised, one CTA per SM (192 threads):
+// Persistent, warp-specialised, one CTA per SM (320 threads):
 //   warp 0      TMA producer: A and B tiles (128 x 64 and BN x 64 bf16, 128-byte
 //               swizzle) into a ring of shared-memory stages;
 //   warp 1      owns the tensor memory and issues tcgen05.mma (M = 128, N = BN,
 //               K = 16) into one of two TMEM accumulators;
-//   warps 2..5  epilogue: tcgen05.ld of the finished accumulator (one row per
-//               thread), the fused epilogue, global stores; the second
-//               accumulator lets the next tile's MMAs run meanwhile.
+//   warps 2..9  epilogue: tcgen05.ld of the finished accumulator (one row per
+//               thread; two warps per TMEM lane quarter, each taking half of
+//               the tile's columns), the fused epilogue, global stores; the
+//               second accumulator lets the next tile's MMAs run meanwhile.
 // Rows beyond M are zero-filled by TMA and never stored.  Requires K % 64 == 0
 // and N % BN == 0 (checked by the launcher).
 #include <cudaTypedefs.h>
@@ -24,8 +25,8 @@ namespace {
 using namespace tc;
 
 constexpr int BM = 128, BK = 64;
-constexpr int kThreads = 192;
-constexpr int kEpiThreads = 128;
+constexpr int kThreads = 320;
+constexpr int kEpiThreads = 256;
 
 template <int BN>
 struct GemmCfg {
@@ -192,6 +193,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   } else {
     // ---------------------------------------------------------- epilogue
     const int q = warp & 3;                 // TMEM lane quarter of this warp
+    const int half = (warp - 2) >> 2;       // which half of the tile's columns
     const int row = q * 32 + lane;
     int it = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++it) {
@@ -203,7 +205,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       const int m = mt * BM + row;
       const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
+      for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
         uint32_t r[32];
         tmem_ld32(tbase + uint32_t(c), r);
         tmem_wait_ld();
