@@ -35,7 +35,11 @@ struct GemmCfg {
   static constexpr int kBBytes = BN * BK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kTmemCols = 2 * BN;           // two accumulators
-  static constexpr size_t kSmem = size_t(kStages) * kStageBytes + 1024 /*align*/ + 256 /*bars*/;
+  // per epilogue warp: a 32 x 32 fp32 chunk, pitch 33 (conflict-free both ways)
+  static constexpr int kStageFloats = 32 * 33;
+  static constexpr size_t kStagingBytes = size_t(kEpiThreads / 32) * kStageFloats * 4;
+  static constexpr size_t kSmem =
+      size_t(kStages) * kStageBytes + kStagingBytes + 1024 /*align*/ + 256 /*bars*/;
 };
 
 struct Smem {
@@ -43,6 +47,24 @@ struct Smem {
   uint32_t tmem_base;
   int abort;
 };
+
+// GELU(z) = z * Phi(z) with Phi from the erfc approximation of Abramowitz &
+// Stegun, Handbook of Mathematical Functions, formula 7.1.26 (absolute error
+// <= 1.5e-7): erfc(x) = t (a1 + t (a2 + t (a3 + t (a4 + t a5)))) exp(-x^2),
+// t = 1 / (1 + p x), x = |z| / sqrt(2) >= 0.  Its error is far below the bf16
+// rounding of the stored output.
+__device__ __forceinline__ float gelu_as7126(float z) {
+  const float x = fabsf(z) * 0.70710678118654752f;
+  float t;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(t) : "f"(fmaf(0.3275911f, x, 1.0f)));
+  float poly = fmaf(t, 1.061405429f, -1.453152027f);
+  poly = fmaf(t, poly, 1.421413741f);
+  poly = fmaf(t, poly, -0.284496736f);
+  poly = fmaf(t, poly, 0.254829592f);
+  const float y = t * poly * ex2(-x * x * 1.4426950408889634f);   // erfc(x)
+  const float phi = z >= 0.f ? fmaf(-0.5f, y, 1.0f) : 0.5f * y;
+  return z * phi;
+}
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
@@ -66,39 +88,65 @@ __device__ __forceinline__ void epilogue32(const EpiArgs& ea, int m, int n, int 
   if constexpr (E == Epi::Bias || E == Epi::BiasGelu) {
     if constexpr (E == Epi::BiasGelu) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) v[j] = gelu_erf(v[j]);
+      for (int j = 0; j < 32; ++j) v[j] = gelu_as7126(v[j]);
     }
     uint4* o = reinterpret_cast<uint4*>(static_cast<bf16*>(ea.out) + size_t(m) * N + n);
 #pragma unroll
     for (int q = 0; q < 4; ++q)
       o[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
                         pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+  }
+}
+
+// Residual epilogues through a per-warp shared-memory transpose: the warp's 32
+// rows x 32 columns of accumulators go to shared memory row by row (one row per
+// thread), then each thread takes one column and the warp walks the 32 rows, so
+// every fp32 load and store of the residual stream covers 128 contiguous bytes.
+// row0: first tile row of this warp; n: first column of the chunk.
+template <Epi E>
+__device__ __forceinline__ void epilogue32_rows(const EpiArgs& ea, int row0, int M, int n, int N,
+                                                const uint32_t (&acc)[32], float* stg,
+                                                int lane) {
+#pragma unroll
+  for (int j = 0; j < 32; ++j) stg[lane * 33 + j] = __uint_as_float(acc[j]);
+  __syncwarp();
+  const int col = n + lane;
+  const float bias = __bfloat162float(static_cast<const bf16*>(ea.bias)[col]);
+  float* out = static_cast<float*>(ea.out);
+  // every load of the chunk is issued before any store (the update is in place)
+  float rv[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i)
+    rv[i] = row0 + i < M ? ea.res[size_t(row0 + i) * N + col] : 0.f;
+  if constexpr (E == Epi::BiasResidual) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (row0 + i < M) out[size_t(row0 + i) * N + col] = rv[i] + (stg[i * 33 + lane] + bias);
   } else {
-    const float4* r = reinterpret_cast<const float4*>(ea.res + size_t(m) * N + n);
-    float4 rv[8];
+    // last sparse block: hn = h + f(h); x'[xrow] = x0 + (hn - h0), h0 == x0.
+    // Element offsets fit 32 bits: sr_create rejects B * L * width >= 2^31.
 #pragma unroll
-    for (int q = 0; q < 8; ++q) rv[q] = r[q];
-    if constexpr (E == Epi::BiasResidual) {
-      float4* o = reinterpret_cast<float4*>(static_cast<float*>(ea.out) + size_t(m) * N + n);
+    for (int half = 0; half < 32; half += 16) {
+      uint32_t xrow[16];
+      float x0[16];
 #pragma unroll
-      for (int q = 0; q < 8; ++q)
-        o[q] = make_float4(rv[q].x + v[4 * q], rv[q].y + v[4 * q + 1], rv[q].z + v[4 * q + 2],
-                           rv[q].w + v[4 * q + 3]);
-    } else {
-      // last sparse block: hn = h + f(h); x'[xrow] = x0 + (hn - h0), h0 == x0
-      const int b = m / ea.Kr;
-      const size_t xrow = size_t(b) * ea.Lx + ea.idx[m];
-      float4* o = reinterpret_cast<float4*>(static_cast<float*>(ea.out) + xrow * N + n);
+      for (int i = 0; i < 16; ++i) {
+        const int m = row0 + half + i < M ? row0 + half + i : row0;
+        xrow[i] = (uint32_t(m / ea.Kr) * uint32_t(ea.Lx) + uint32_t(ea.idx[m])) * uint32_t(N) +
+                  uint32_t(col);
+      }
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const float4 x0 = o[q];
-        const float hn[4] = {rv[q].x + v[4 * q], rv[q].y + v[4 * q + 1], rv[q].z + v[4 * q + 2],
-                             rv[q].w + v[4 * q + 3]};
-        o[q] = make_float4(x0.x + (hn[0] - x0.x), x0.y + (hn[1] - x0.y), x0.z + (hn[2] - x0.z),
-                           x0.w + (hn[3] - x0.w));
+      for (int i = 0; i < 16; ++i) x0[i] = row0 + half + i < M ? out[xrow[i]] : 0.f;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        if (row0 + half + i < M) {
+          const float hn = rv[half + i] + (stg[(half + i) * 33 + lane] + bias);
+          out[xrow[i]] = x0[i] + (hn - x0[i]);
+        }
       }
     }
   }
+  __syncwarp();
 }
 
 template <int BN, Epi E>
@@ -111,7 +159,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* sA = base;
   unsigned char* sB = base + size_t(C::kStages) * C::kABytes;
-  Smem* sm = reinterpret_cast<Smem*>(base + size_t(C::kStages) * C::kStageBytes);
+  float* staging = reinterpret_cast<float*>(base + size_t(C::kStages) * C::kStageBytes);
+  Smem* sm = reinterpret_cast<Smem*>(base + size_t(C::kStages) * C::kStageBytes +
+                                     C::kStagingBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int m_tiles = (M + BM - 1) / BM;
@@ -141,7 +191,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       uint32_t phase = 0;
       uint32_t issued = 0, issued_phase = 0;    // per stage: loads in flight, their parity
       for (int t = blockIdx.x; t < tiles && !*abort; t += gridDim.x) {
-        const int mt = t % m_tiles, nt = t / m_tiles;
+        const int nt = t % n_tiles, mt = t / n_tiles;
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait(&sm->empty[stage], phase ^ 1, abort, ea.fault)) break;
           mbar_arrive_expect_tx(&sm->full[stage], C::kStageBytes);
@@ -197,7 +247,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const int row = q * 32 + lane;
     int it = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++it) {
-      const int mt = t % m_tiles, nt = t / m_tiles;
+      const int nt = t % n_tiles, mt = t / n_tiles;
       const int acc = it & 1;
       const uint32_t aphase = (it >> 1) & 1;
       if (!__all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault))) break;
@@ -209,7 +259,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         uint32_t r[32];
         tmem_ld32(tbase + uint32_t(c), r);
         tmem_wait_ld();
-        if (m < M) epilogue32<E>(ea, m, nt * BN + c, N, r);
+        if constexpr (E == Epi::Bias || E == Epi::BiasGelu) {
+          if (m < M) epilogue32<E>(ea, m, nt * BN + c, N, r);
+        } else {
+          epilogue32_rows<E>(ea, mt * BM + q * 32, M, nt * BN + c, N, r,
+                             staging + (warp - 2) * C::kStageFloats, lane);
+        }
       }
       tc_fence_before();
       mbar_arrive(&sm->tempty[acc]);
