@@ -27,6 +27,14 @@ if ROOT not in sys.path:
 DEFAULT_WORKLOAD = "c4_0p25deg_bf16"
 L2_FLUSH_BYTES = 512 << 20          # > 129 MB of L2
 
+# DRAM bytes (read + write) per launch of a kernel kind on a workload, from one
+# ncu capture of the current kernel (profiles/attention_tc_c4_*.md): the 0.25 deg
+# forward runs 8 dense attention launches (114.4 MB each) and 16 sparse ones
+# (24.9 MB each).  None when no capture of the current kernel exists.
+DRAM_TRAFFIC_PER_LAUNCH = {
+    ("attention", "c4_0p25deg_bf16"): (8 * 114.4e6 + 16 * 24.9e6) / 24,
+}
+
 
 def _peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -210,7 +218,7 @@ def run_ours(args, rank, world, local_rank):
     return wl, K, ms, wall, clk, trace, e2e_ms, bytes_io
 
 
-def roofline(trace, peaks, steps):
+def roofline(trace, peaks, steps, workload):
     kernels = {k: v for k, v in trace.items() if k != "copy" and v["launches"] > 0}
     dom = max(kernels, key=lambda k: kernels[k]["ms"])
     t = kernels[dom]
@@ -235,10 +243,12 @@ def roofline(trace, peaks, steps):
         detail[k] = d
     return ({"kernel": dom, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
              "frac": achieved / peak, "peak_source": peaks["source"] +
-             (" sustained" if bound == "tensor" else ""), "traffic": None}, detail)
+             (" sustained" if bound == "tensor" else ""),
+             "traffic": DRAM_TRAFFIC_PER_LAUNCH.get((dom, workload)),
+             "algorithmic_bytes_per_launch": t["bytes"] / t["launches"]}, detail)
 
 
-def cpu_baseline(wl, budget_s=25.0):
+def cpu_baseline(wl, sparse_only=False):
     """The fp64 oracle, as it stands, on a bounded sample of the workload: one dense
     block over all L tokens and one sparse block over the K routed tokens of the
     same model; the full forward's time is those block times weighted by the
@@ -254,9 +264,11 @@ def cpu_baseline(wl, budget_s=25.0):
     K = o.keep_count(wl.L, wl.keep_ratio)
     from concurrent.futures import ThreadPoolExecutor
     pool = ThreadPoolExecutor(threads)
-    t0 = time.perf_counter()
-    o.block(x, w, wl.heads, pool=pool)
-    t_dense = time.perf_counter() - t0
+    t_dense = 0.0
+    if not sparse_only:
+        t0 = time.perf_counter()
+        o.block(x, w, wl.heads, pool=pool)
+        t_dense = time.perf_counter() - t0
     idx = o.select_random(wl.B, wl.L, K, 1)
     h = x[np.arange(wl.B)[:, None], idx]
     t0 = time.perf_counter()
@@ -310,7 +322,7 @@ def main():
     peaks = _peaks()
     tokens = wl.B * wl.L * world
     value = tokens / (ms * 1e-3)
-    roof, detail = roofline(trace, peaks, args.steps)
+    roof, detail = roofline(trace, peaks, args.steps, wl.name)
     launches = sum(v["launches"] for v in trace.values())
     gs = {}
     for k in ("gather", "gemm_fc2_scatter"):
@@ -352,10 +364,12 @@ def run_reference(args, rank, world):
     K = o.keep_count(wl.L, wl.keep_ratio)
     vals = []
     base = None
-    for i in range(args.warmup + args.steps):
+    # untimed warm-up steps run the cheap half of the sample (one sparse block)
+    for i in range(args.warmup):
+        cpu_baseline(wl, sparse_only=True)
+    for i in range(args.steps):
         base = cpu_baseline(wl)
-        if i >= args.warmup:
-            vals.append(base["value"])
+        vals.append(base["value"])
     value = sum(vals) / len(vals)
     ms = wl.B * wl.L / value * 1e3
     line = {"impl": "reference", "metric": "full-grid tokens/sec of routed encoder fwd",

@@ -7,18 +7,17 @@
 // One CTA owns 256 query rows of one (sample, head) as two 128-row tiles that
 // share every K/V tile, 384 threads:
 //   warps 0, 3  TMA: the two Q tiles once, then K_j (warp 0) and V_j (warp 3),
-//               128 keys x 64, into two 2-stage rings (3-D tensor map over
+//               128 keys x 64, into two 3-stage rings (3-D tensor map over
 //               [B, T, 3D], zero fill past T); a K stage frees as soon as both
 //               tiles' S MMAs that read it finish, a V stage when the P V MMAs do;
 //   warps 1, 2  tcgen05.mma for tile 0 and tile 1, each thread in its own order:
 //               S^t = Q^t K_j^T (128 x 128, fp32 in TMEM), O^t += P^t V_j
-//               (128 x 64, accumulated in TMEM); the next S^t is issued as soon
-//               as softmax t has read the current one;
+//               (128 x 64, accumulated in TMEM, P from TMEM); the next S^t is
+//               issued as soon as softmax t has read the current one;
 //   warps 4-7   softmax of tile 0, warps 8-11 softmax of tile 1: one query row
 //               per thread.  Each reads its S row from TMEM, updates the
-//               running max and sum, writes P = 2^(s*c - m*c) as bf16 into one
-//               of two 128B-swizzled shared tiles (the A operand of the P V
-//               MMA), so P of the next key tile never waits for this P V.
+//               running max and sum, and writes P = 2^(s*c - m*c) as bf16
+//               pairs into tensor memory, where the P V MMA reads its A operand.
 // The running max is only raised when it grows by more than 2^8 (in the exp2
 // domain); then the thread rescales its O row in TMEM first.  P, O and the sum
 // always use the same max, so the result is exact up to rounding.
@@ -36,27 +35,27 @@ using namespace tc;
 constexpr int kDh = 64;
 constexpr int kQTile = 128, kQTiles = 2, kBQ = kQTile * kQTiles;
 constexpr int kKV = 128;
-constexpr int kStages = 2;                                    // K ring and V ring
+constexpr int kStages = 3;                                    // K ring and V ring
 constexpr int kThreads = 384;
 constexpr int kTileBytes = kQTile * kDh * 2;                  // 16 KB: 128 rows x 128 B
-constexpr int kPBytes = kQTile * kKV * 2;                     // 32 KB: two 64-key atoms
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColS = 0;      // S^t at columns [128 t, 128 t + 128)
 constexpr uint32_t kColO = 256;    // O^t at columns [256 + 64 t, 256 + 64 t + 64)
+constexpr uint32_t kColP = 384;    // P^t (bf16 pairs) at columns [384 + 64 t, 384 + 64 t + 64)
 // raise the running max only when it grows by more than 8 in the exp2 domain
 constexpr float kRescaleLog2 = 8.0f;
 
 struct AttSmem {
   uint64_t q_full;
   uint64_t k_full[kStages], k_empty[kStages], v_full[kStages], v_empty[kStages];
-  uint64_t s_full[kQTiles], s_free[kQTiles], p_full[kQTiles][2], pv_done[kQTiles][2];
+  uint64_t s_full[kQTiles], s_free[kQTiles], p_full[kQTiles], pv_done[kQTiles];
   uint64_t drain[kQTiles];
   uint32_t tmem_base;
   int abort;
 };
 
 constexpr size_t kSmemBytes = 1024 /*align*/ + size_t(kQTiles) * kTileBytes +
-                              size_t(kStages) * 2 * kTileBytes + size_t(kQTiles) * 2 * kPBytes + 256;
+                              size_t(kStages) * 2 * kTileBytes + 256;
 
 // packed fp32 pairs (the f32x2 instructions of sm_100+)
 __device__ __forceinline__ uint64_t pk2(float lo, float hi) {
@@ -90,10 +89,9 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* sQ = base;                                  // 2 x 16 KB
-  unsigned char* sK = sQ + kQTiles * kTileBytes;             // 2 stages x 16 KB
-  unsigned char* sV = sK + kStages * kTileBytes;             // 2 stages x 16 KB
-  unsigned char* sP = sV + kStages * kTileBytes;             // [tile][buffer] x 32 KB
-  AttSmem* sm = reinterpret_cast<AttSmem*>(sP + kQTiles * 2 * kPBytes);
+  unsigned char* sK = sQ + kQTiles * kTileBytes;             // stages x 16 KB
+  unsigned char* sV = sK + kStages * kTileBytes;             // stages x 16 KB
+  AttSmem* sm = reinterpret_cast<AttSmem*>(sV + kStages * kTileBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qblocks = (T + kBQ - 1) / kBQ;
@@ -114,10 +112,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
     for (int t = 0; t < kQTiles; ++t) {
       mbar_init(&sm->s_full[t], 1);
       mbar_init(&sm->s_free[t], kQTile);
-      for (int bf = 0; bf < 2; ++bf) {
-        mbar_init(&sm->p_full[t][bf], kQTile);
-        mbar_init(&sm->pv_done[t][bf], 1);
-      }
+      mbar_init(&sm->p_full[t], kQTile);
+      mbar_init(&sm->pv_done[t], 1);
       mbar_init(&sm->drain[t], 1);
     }
     sm->abort = 0;
@@ -146,15 +142,16 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
       unsigned char* ring = is_k ? sK : sV;
       const int col = (is_k ? D : 2 * D) + h * kDh;
       uint32_t issued = 0, par = 0;   // stages holding a load; parity of its phase
+      int st = 0;
+      uint32_t ph = 0;
       for (int j = 0; j < nkv; ++j) {
-        const int st = j & 1;
-        const uint32_t ph = (j >> 1) & 1;
-        // the stage is free once both tiles' MMAs of key tile j - 2 have read it
+        // the stage is free once both tiles' MMAs of key tile j - kStages have read it
         if (!mbar_wait(&empty[st], ph ^ 1, abort, fault)) break;
         mbar_arrive_expect_tx(&full[st], kTileBytes);
         tma_load_3d(&tm, ring + st * kTileBytes, &full[st], col, j * kKV, b);
         issued |= 1u << st;
         par = (par & ~(1u << st)) | (ph << st);
+        if (++st == kStages) { st = 0; ph ^= 1; }
       }
       // every issued load lands before the CTA may exit
       int no_abort = 0;
@@ -186,28 +183,31 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
         tc_fence_after();
         issue_s(0);
       }
+      const uint32_t aP = tmem + kColP + uint32_t(t * (kKV / 2));
+      int vs = 0;                 // stage of V_j
+      uint32_t vph = 0;
       for (int j = 0; j < nkv && ok; ++j) {
         // S for the next key tile as soon as the softmax has read this one
         if (j + 1 < nkv) {
-          const int st = (j + 1) & 1;
-          if (!(ok = mbar_wait(&sm->k_full[st], ((j + 1) >> 1) & 1, abort, fault))) break;
+          const int st = vs + 1 == kStages ? 0 : vs + 1;
+          const uint32_t sph = vs + 1 == kStages ? vph ^ 1 : vph;
+          if (!(ok = mbar_wait(&sm->k_full[st], sph, abort, fault))) break;
           if (!(ok = mbar_wait(&sm->s_free[t], j & 1, abort, fault))) break;
           tc_fence_after();
           issue_s(st);
         }
-        // O^t += P^t_j V_j
-        const int vs = j & 1;
-        if (!(ok = mbar_wait(&sm->v_full[vs], (j >> 1) & 1, abort, fault))) break;
-        if (!(ok = mbar_wait(&sm->p_full[t][j & 1], (j >> 1) & 1, abort, fault))) break;
+        // O^t += P^t_j V_j with P read from tensor memory (64 columns of bf16 pairs)
+        if (!(ok = mbar_wait(&sm->v_full[vs], vph, abort, fault))) break;
+        if (!(ok = mbar_wait(&sm->p_full[t], j & 1, abort, fault))) break;
         tc_fence_after();
-        const uint32_t pa = smem_u32(sP + (t * 2 + (j & 1)) * kPBytes);
         const uint32_t va = smem_u32(sV + vs * kTileBytes);
 #pragma unroll
         for (int k = 0; k < kKV / 16; ++k)
-          mma_bf16(dO, sw128_desc(pa + (k >> 2) * (kQTile * 128) + (k & 3) * 32),
-                   sw128_desc_mn(va + k * 2048), idesc_o, (j | k) != 0 ? 1u : 0u);
-        mma_commit(&sm->pv_done[t][j & 1]);
+          mma_bf16_ts(dO, aP + uint32_t(k * 8), sw128_desc_mn(va + k * 2048), idesc_o,
+                      (j | k) != 0 ? 1u : 0u);
+        mma_commit(&sm->pv_done[t]);
         mma_commit(&sm->v_empty[vs]);
+        if (++vs == kStages) { vs = 0; vph ^= 1; }
       }
       int no_abort = 0;
       mma_commit(&sm->drain[t]);
@@ -221,6 +221,7 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
     const uint32_t lane_off = uint32_t(quarter * 32) << 16;
     const uint32_t tS = tmem + lane_off + kColS + uint32_t(t * kKV);
     const uint32_t tO = tmem + lane_off + kColO + uint32_t(t * kDh);
+    const uint32_t tP = tmem + lane_off + kColP + uint32_t(t * (kKV / 2));
     const float c = 0.125f * 1.4426950408889634f;  // 1/sqrt(64) * log2(e)
     const float thresh = kRescaleLog2 / c;         // the same threshold in score units
     const uint64_t c2 = pk2(c, c);
@@ -268,24 +269,23 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
         l_run *= alpha;
         rescale = true;
       }
-      // P buffer j % 2 was last read by P V of tile j - 2
-      if (j >= 2) {
-        ok = __all_sync(0xffffffffu,
-                        mbar_wait(&sm->pv_done[t][j & 1], ((j >> 1) & 1) ^ 1, abort, fault));
+      // P and O of this tile are free once the previous P V has completed
+      if (j >= 1) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (j - 1) & 1, abort, fault));
         if (!ok) break;
+        tc_fence_after();
       }
-      // P = 2^(s c - m c) as bf16 into the 128B-swizzled K-major tile: 16-byte
-      // chunk cc of the row goes to atom cc / 8, slot (cc % 8) ^ (r % 8)
-      unsigned char* prow = sP + (t * 2 + (j & 1)) * kPBytes + r * 128;
+      // P = 2^(s c - m c) as bf16 pairs into tensor memory: key 2i and 2i+1 of
+      // this row share column i of the tile's P region (the A operand of P V)
       const float mc = m_run * c;
       const uint64_t nmc2 = pk2(-mc, -mc);
       uint64_t ls2[2] = {pk2(0.f, 0.f), pk2(0.f, 0.f)};
 #pragma unroll
-      for (int cc = 0; cc < kKV / 8; ++cc) {
-        uint32_t w[4];
+      for (int cc = 0; cc < kKV / 32; ++cc) {
+        uint32_t w[16];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int i0 = 8 * cc + 2 * q;
+        for (int q = 0; q < 16; ++q) {
+          const int i0 = 32 * cc + 2 * q;
           const uint64_t arg = fma2(pk2(__uint_as_float(s[i0 / 32][i0 % 32]),
                                         __uint_as_float(s[(i0 + 1) / 32][(i0 + 1) % 32])),
                                     c2, nmc2);
@@ -295,9 +295,7 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
           ls2[q & 1] = add2(ls2[q & 1], pk2(p0, p1));
           w[q] = pack_bf16x2(p0, p1);
         }
-        const int atom = cc >> 3, slot = (cc & 7) ^ (r & 7);
-        *reinterpret_cast<uint4*>(prow + atom * (kQTile * 128) + slot * 16) =
-            make_uint4(w[0], w[1], w[2], w[3]);
+        tmem_st16(tP + uint32_t(cc * 16), w);
       }
       {
         float l0, l1, l2, l3;
@@ -305,12 +303,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
         up2(ls2[1], l2, l3);
         l_run += (l0 + l1) + (l2 + l3);
       }
-      // a raised max rescales O, which then holds every earlier P V product
+      // a raised max rescales O, which holds every earlier P V product
       if (__any_sync(0xffffffffu, rescale)) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t][(j - 1) & 1],
-                                               ((j - 1) >> 1) & 1, abort, fault));
-        if (!ok) break;
-        tc_fence_after();
         uint32_t o[32];
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
@@ -320,16 +314,13 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
           for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
           tmem_st32(tO + uint32_t(half * 32), o);
         }
-        tmem_wait_st();
       }
-      fence_proxy_async_smem();
+      tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&sm->p_full[t][j & 1]);
+      mbar_arrive(&sm->p_full[t]);
     }
     // epilogue: O / l for the rows that exist (the last P V implies all earlier ones)
-    if (ok)
-      ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t][(nkv - 1) & 1],
-                                             ((nkv - 1) >> 1) & 1, abort, fault));
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (nkv - 1) & 1, abort, fault));
     if (ok) {
       tc_fence_after();
       uint32_t o[2][32];
