@@ -88,7 +88,7 @@ class ClockSampler:
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=self.fh, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
@@ -288,13 +288,15 @@ def cpu_baseline(wl, sparse_only=False):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--split", default=None,
                     help="override the block split n1,n2,n3 (kernel studies and profiling)")
+    ap.add_argument("--sweep", choices=["gather"], default=None,
+                    help="size sweep of one kernel (prints one JSON line per size)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -304,6 +306,8 @@ def main():
 
     if args.impl == "reference":
         return run_reference(args, rank, world)
+    if args.sweep == "gather":
+        return gather_sweep(args)
 
     import torch
     import torch.distributed as dist
@@ -353,6 +357,45 @@ def main():
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def gather_sweep(args):
+    """Gather GB/s from 33 MB to 4.2 GB moved: one sparse block (split 0,1,0) of the
+    0.25 deg model (L=16200, D=1024, r=0.25) at batch 1..128, L2 flushed before
+    every traced forward; the gather kernel's CUDA-event time from the trace."""
+    import torch
+    from paper_2607_02829_gb300 import binding as b, build, synth
+    build.build()
+    peaks = _peaks()
+    L, D, H, r = 16200, 1024, 16, 0.25
+    w = {k: synth.to_storage(v, "bf16").cuda()
+         for k, v in synth.make_block_weights(D, 4 * D, 7).items()}
+    warr = b.weights_array([w])
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    s = torch.cuda.current_stream()
+    for B in (1, 2, 4, 8, 16, 32, 64, 128):
+        cfg = b.make_config(B, L, D, H, 0, 1, 0, dtype="bf16")
+        enc = b.Encoder(cfg, max_keep_ratio=r)
+        x = torch.randn(B, L, D, device="cuda").to(torch.bfloat16)
+        out = torch.empty_like(x)
+        for i in range(args.warmup):
+            b.sr_forward(enc.handle, x.data_ptr(), warr, r, i, out.data_ptr(), None, s.cuda_stream)
+        b.sr_trace_enable(enc.handle, True)
+        b.sr_trace_read(enc.handle, reset=True)
+        for i in range(args.steps):
+            flush.zero_()
+            b.sr_forward(enc.handle, x.data_ptr(), warr, r, 100 + i, out.data_ptr(), None,
+                         s.cuda_stream)
+        torch.cuda.synchronize()
+        t = b.sr_trace_read(enc.handle, reset=True)["gather"]
+        gbs = t["bytes"] / (t["ms"] * 1e-3) / 1e9
+        print(json.dumps({"sweep": "gather", "B": B, "rows": B * b.sr_keep_count(L, r),
+                          "bytes_per_launch": t["bytes"] / t["launches"],
+                          "us_per_launch": t["ms"] / t["launches"] * 1e3, "gbs": gbs,
+                          "frac_of_hbm": gbs / peaks["hbm_gbs"]}), flush=True)
+        enc.close()
+        del x, out
+        torch.cuda.empty_cache()
 
 
 def run_reference(args, rank, world):

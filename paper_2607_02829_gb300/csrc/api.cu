@@ -62,6 +62,7 @@ size_t elem_size(int32_t dtype) { return dtype == SR_BF16 ? 2 : 4; }
 // Workspace layout for a config and a maximum routed count Kmax.
 struct Plan {
   size_t fault, xs, ln, qkv, att, u, hs, idx, score, total;
+  size_t block_rows;   // rows the per-block buffers (ln, qkv, att, u) hold
 };
 
 Plan make_plan(const sr_config& c, int32_t Kmax) {
@@ -69,13 +70,17 @@ Plan make_plan(const sr_config& c, int32_t Kmax) {
   const size_t rows = size_t(c.B) * c.L;
   const size_t rrows = size_t(c.B) * (Kmax > 0 ? Kmax : 0);
   Plan p{};
+  // dense blocks (or the r = 1 path) see all B*L rows; a model that is only a
+  // sparse stage, used with keep ratios below 1, sees at most B*Kmax
+  p.block_rows = (c.n1 + c.n3 > 0 || Kmax >= c.L) ? rows : rrows;
+  const size_t brows = p.block_rows;
   size_t off = 0;
   p.fault = off; off += kAlign;                                   // device fault word
   p.xs = off;    off += align_up(rows * c.D * sizeof(float));     // fp32 residual stream
-  p.ln = off;    off += align_up(rows * c.D * es);
-  p.qkv = off;   off += align_up(rows * 3 * c.D * es);
-  p.att = off;   off += align_up(rows * c.D * es);
-  p.u = off;     off += align_up(rows * size_t(c.mlp_hidden) * es);
+  p.ln = off;    off += align_up(brows * c.D * es);
+  p.qkv = off;   off += align_up(brows * 3 * c.D * es);
+  p.att = off;   off += align_up(brows * c.D * es);
+  p.u = off;     off += align_up(brows * size_t(c.mlp_hidden) * es);
   p.hs = off;    off += align_up(rrows * c.D * sizeof(float));    // fp32 routed stream
   p.idx = off;   off += align_up(size_t(c.B) * c.L * sizeof(int32_t));
   p.score = off; off += align_up(rows * sizeof(float));
@@ -353,6 +358,8 @@ sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, flo
   const bool route = keep_ratio < 1.0f && c.n2 > 0;
   if (K < 1 && (route || idx_out)) return fail(SR_ERR_INVALID_ARG, "K = floor(L * keep_ratio) is 0");
   if (route && K > h->Kmax) return fail(SR_ERR_WORKSPACE, "K exceeds the workspace's routed capacity");
+  if (!route && c.n2 > 0 && size_t(c.B) * c.L > h->plan.block_rows)
+    return fail(SR_ERR_WORKSPACE, "workspace sized for keep ratios below 1 only");
   const size_t bytes = size_t(c.B) * c.L * c.D * h->es;
   const char* xb = static_cast<const char*>(x);
   char* ob = static_cast<char*>(out);

@@ -9,8 +9,10 @@
 //               K = 16) into one of two TMEM accumulators;
 //   warps 2..9  epilogue: tcgen05.ld of the finished accumulator (one row per
 //               thread; two warps per TMEM lane quarter, each taking half of
-//               the tile's columns), the fused epilogue, global stores; the
-//               second accumulator lets the next tile's MMAs run meanwhile.
+//               the tile's columns), the fused epilogue, then a per-warp
+//               shared-memory transpose so that every global load and store
+//               covers whole row segments; the second accumulator lets the
+//               next tile's MMAs run meanwhile.
 // Rows beyond M are zero-filled by TMA and never stored.  Requires K % 64 == 0
 // and N % BN == 0 (checked by the launcher).
 #include <cudaTypedefs.h>
@@ -69,33 +71,48 @@ __device__ __forceinline__ float gelu_as7126(float z) {
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
-// Epilogue of 32 consecutive columns n..n+31 of row m (acc in fp32 bits).
-template <Epi E>
-__device__ __forceinline__ void epilogue32(const EpiArgs& ea, int m, int n, int N,
-                                           const uint32_t (&acc)[32]) {
+// bf16 epilogues (bias; bias + GELU) over W = 64 or 32 consecutive columns
+// n..n+W-1 of the warp's 32 rows row0..row0+31: each thread biases (and GELUs)
+// its own row and packs it into W/2 bf16 pairs in shared memory, then the warp
+// writes the chunk row by row, so every store covers 2W contiguous bytes.
+template <Epi E, int W>
+__device__ __forceinline__ void epilogue_bf16(const EpiArgs& ea, int row0, int M, int n, int N,
+                                              const uint32_t (&acc)[W / 32][32], uint32_t* stg,
+                                              int lane) {
   const uint4* bias4 = reinterpret_cast<const uint4*>(static_cast<const bf16*>(ea.bias) + n);
-  float v[32];
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
+  for (int q = 0; q < W / 8; ++q) {
     const uint4 bq = __ldg(bias4 + q);
     const uint32_t bw[4] = {bq.x, bq.y, bq.z, bq.w};
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      v[8 * q + 2 * j] = __uint_as_float(acc[8 * q + 2 * j]) + bf16_lo(bw[j]);
-      v[8 * q + 2 * j + 1] = __uint_as_float(acc[8 * q + 2 * j + 1]) + bf16_hi(bw[j]);
+      const int c0 = 8 * q + 2 * j;
+      float v0 = __uint_as_float(acc[c0 / 32][c0 % 32]) + bf16_lo(bw[j]);
+      float v1 = __uint_as_float(acc[(c0 + 1) / 32][(c0 + 1) % 32]) + bf16_hi(bw[j]);
+      if constexpr (E == Epi::BiasGelu) {
+        v0 = gelu_as7126(v0);
+        v1 = gelu_as7126(v1);
+      }
+      stg[lane * 33 + 4 * q + j] = pack_bf16x2(v0, v1);
     }
   }
-  if constexpr (E == Epi::Bias || E == Epi::BiasGelu) {
-    if constexpr (E == Epi::BiasGelu) {
-#pragma unroll
-      for (int j = 0; j < 32; ++j) v[j] = gelu_as7126(v[j]);
+  __syncwarp();
+  uint32_t* out = static_cast<uint32_t*>(ea.out);        // bf16 pairs
+  const int ldw = N / 2;
+  if constexpr (W == 64) {
+#pragma unroll 8
+    for (int i = 0; i < 32; ++i)
+      if (row0 + i < M) out[size_t(row0 + i) * ldw + n / 2 + lane] = stg[i * 33 + lane];
+  } else {
+    // 16 pairs per row: half a warp per row, two rows per store
+#pragma unroll 8
+    for (int i = 0; i < 32; i += 2) {
+      const int rr = i + (lane >> 4);
+      if (row0 + rr < M)
+        out[size_t(row0 + rr) * ldw + n / 2 + (lane & 15)] = stg[rr * 33 + (lane & 15)];
     }
-    uint4* o = reinterpret_cast<uint4*>(static_cast<bf16*>(ea.out) + size_t(m) * N + n);
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      o[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
-                        pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
   }
+  __syncwarp();
 }
 
 // Residual epilogues through a per-warp shared-memory transpose: the warp's 32
@@ -103,21 +120,25 @@ __device__ __forceinline__ void epilogue32(const EpiArgs& ea, int m, int n, int 
 // thread), then each thread takes one column and the warp walks the 32 rows, so
 // every fp32 load and store of the residual stream covers 128 contiguous bytes.
 // row0: first tile row of this warp; n: first column of the chunk.
+// The residual rows of a chunk, one column per thread (loads issued together).
+__device__ __forceinline__ void load_residual(const EpiArgs& ea, int row0, int M, int n, int N,
+                                              int lane, float (&rv)[32]) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i)
+    rv[i] = row0 + i < M ? ea.res[size_t(row0 + i) * N + n + lane] : 0.f;
+}
+
 template <Epi E>
 __device__ __forceinline__ void epilogue32_rows(const EpiArgs& ea, int row0, int M, int n, int N,
-                                                const uint32_t (&acc)[32], float* stg,
-                                                int lane) {
+                                                const uint32_t (&acc)[32], const float (&rv)[32],
+                                                float* stg, int lane) {
 #pragma unroll
   for (int j = 0; j < 32; ++j) stg[lane * 33 + j] = __uint_as_float(acc[j]);
   __syncwarp();
   const int col = n + lane;
   const float bias = __bfloat162float(static_cast<const bf16*>(ea.bias)[col]);
   float* out = static_cast<float*>(ea.out);
-  // every load of the chunk is issued before any store (the update is in place)
-  float rv[32];
-#pragma unroll
-  for (int i = 0; i < 32; ++i)
-    rv[i] = row0 + i < M ? ea.res[size_t(row0 + i) * N + col] : 0.f;
+  // the residual of the chunk was loaded before (the update is in place)
   if constexpr (E == Epi::BiasResidual) {
 #pragma unroll
     for (int i = 0; i < 32; ++i)
@@ -244,26 +265,43 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // ---------------------------------------------------------- epilogue
     const int q = warp & 3;                 // TMEM lane quarter of this warp
     const int half = (warp - 2) >> 2;       // which half of the tile's columns
-    const int row = q * 32 + lane;
+    constexpr int kW = BN / 2 >= 64 ? 64 : 32;    // bf16 epilogue step (columns)
     int it = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++it) {
       const int nt = t % n_tiles, mt = t / n_tiles;
       const int acc = it & 1;
       const uint32_t aphase = (it >> 1) & 1;
-      if (!__all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault))) break;
-      tc_fence_after();
-      const int m = mt * BM + row;
-      const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
+      const int row0 = mt * BM + q * 32;
+      const int c_begin = half * (BN / 2), c_end = (half + 1) * (BN / 2);
+      if constexpr (E == Epi::Bias || E == Epi::BiasGelu) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault))) break;
+        tc_fence_after();
+        const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
 #pragma unroll 1
-      for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
-        uint32_t r[32];
-        tmem_ld32(tbase + uint32_t(c), r);
-        tmem_wait_ld();
-        if constexpr (E == Epi::Bias || E == Epi::BiasGelu) {
-          if (m < M) epilogue32<E>(ea, m, nt * BN + c, N, r);
-        } else {
-          epilogue32_rows<E>(ea, mt * BM + q * 32, M, nt * BN + c, N, r,
+        for (int c = c_begin; c < c_end; c += kW) {
+          uint32_t r[kW / 32][32];
+#pragma unroll
+          for (int k = 0; k < kW / 32; ++k) tmem_ld32(tbase + uint32_t(c + 32 * k), r[k]);
+          tmem_wait_ld();
+          epilogue_bf16<E, kW>(ea, row0, M, nt * BN + c, N, r,
+                               reinterpret_cast<uint32_t*>(staging) + (warp - 2) * C::kStageFloats,
+                               lane);
+        }
+      } else {
+        // the first chunk's residual loads overlap the wait for the accumulator
+        float rv[32];
+        load_residual(ea, row0, M, nt * BN + c_begin, N, lane, rv);
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault))) break;
+        tc_fence_after();
+        const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
+#pragma unroll 1
+        for (int c = c_begin; c < c_end; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(tbase + uint32_t(c), r);
+          tmem_wait_ld();
+          epilogue32_rows<E>(ea, row0, M, nt * BN + c, N, r, rv,
                              staging + (warp - 2) * C::kStageFloats, lane);
+          if (c + 32 < c_end) load_residual(ea, row0, M, nt * BN + c + 32, N, lane, rv);
         }
       }
       tc_fence_before();

@@ -105,3 +105,22 @@ def test_status_strings(L):
     from paper_2607_02829_gb300 import binding as b
     for s in range(6):
         assert L.sr_status_string(s).decode().startswith("SR_")
+
+
+def test_routed_only_workspace_is_smaller_and_rejects_the_dense_path(L):
+    from paper_2607_02829_gb300 import binding as b
+    cfg = b.make_config(2, 512, 256, 4, 0, 2, 0, dtype="f32")
+    small = b.sr_workspace_bytes(cfg, 0.25)
+    full = b.sr_workspace_bytes(cfg, 1.0)
+    assert 0 < small < full
+    h = _handle(b, cfg, small)
+    try:
+        w = (b.sr_block_weights * 2)()
+        for i in range(2):
+            for f in b.WEIGHT_FIELDS:
+                setattr(w[i], f, 0x200000)
+        with pytest.raises(b.SRError) as e:
+            b.sr_forward(h, 0x400000, w, 1.0, 0, 0x800000, None, None)
+        assert e.value.status == b.SR_ERR_WORKSPACE
+    finally:
+        b.sr_destroy(h)
