@@ -54,18 +54,25 @@ struct Smem {
 // Stegun, Handbook of Mathematical Functions, formula 7.1.26 (absolute error
 // <= 1.5e-7): erfc(x) = t (a1 + t (a2 + t (a3 + t (a4 + t a5)))) exp(-x^2),
 // t = 1 / (1 + p x), x = |z| / sqrt(2) >= 0.  Its error is far below the bf16
-// rounding of the stored output.
-__device__ __forceinline__ float gelu_as7126(float z) {
-  const float x = fabsf(z) * 0.70710678118654752f;
-  float t;
-  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(t) : "f"(fmaf(0.3275911f, x, 1.0f)));
-  float poly = fmaf(t, 1.061405429f, -1.453152027f);
-  poly = fmaf(t, poly, 1.421413741f);
-  poly = fmaf(t, poly, -0.284496736f);
-  poly = fmaf(t, poly, 0.254829592f);
-  const float y = t * poly * ex2(-x * x * 1.4426950408889634f);   // erfc(x)
-  const float phi = z >= 0.f ? fmaf(-0.5f, y, 1.0f) : 0.5f * y;
-  return z * phi;
+// rounding of the stored output.  Two values at once, with the packed fp32
+// instructions.
+__device__ __forceinline__ void gelu2_as7126(float& z0, float& z1) {
+  const uint64_t x = mul2(pk2(fabsf(z0), fabsf(z1)),
+                          pk2(0.70710678118654752f, 0.70710678118654752f));
+  float d0, d1;
+  up2(fma2(x, pk2(0.3275911f, 0.3275911f), pk2(1.0f, 1.0f)), d0, d1);
+  const uint64_t t = pk2(rcp_approx(d0), rcp_approx(d1));
+  uint64_t poly = fma2(t, pk2(1.061405429f, 1.061405429f), pk2(-1.453152027f, -1.453152027f));
+  poly = fma2(t, poly, pk2(1.421413741f, 1.421413741f));
+  poly = fma2(t, poly, pk2(-0.284496736f, -0.284496736f));
+  poly = fma2(t, poly, pk2(0.254829592f, 0.254829592f));
+  float a0, a1;
+  up2(mul2(mul2(x, x), pk2(-1.4426950408889634f, -1.4426950408889634f)), a0, a1);
+  // 0.5 erfc(|z| / sqrt 2) = Phi(-|z|)
+  float h0, h1;
+  up2(mul2(mul2(mul2(t, poly), pk2(ex2(a0), ex2(a1))), pk2(0.5f, 0.5f)), h0, h1);
+  const uint64_t phi = pk2(z0 >= 0.f ? 1.0f - h0 : h0, z1 >= 0.f ? 1.0f - h1 : h1);
+  up2(mul2(pk2(z0, z1), phi), z0, z1);
 }
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
@@ -89,10 +96,7 @@ __device__ __forceinline__ void epilogue_bf16(const EpiArgs& ea, int row0, int M
       const int c0 = 8 * q + 2 * j;
       float v0 = __uint_as_float(acc[c0 / 32][c0 % 32]) + bf16_lo(bw[j]);
       float v1 = __uint_as_float(acc[(c0 + 1) / 32][(c0 + 1) % 32]) + bf16_hi(bw[j]);
-      if constexpr (E == Epi::BiasGelu) {
-        v0 = gelu_as7126(v0);
-        v1 = gelu_as7126(v1);
-      }
+      if constexpr (E == Epi::BiasGelu) gelu2_as7126(v0, v1);
       stg[lane * 33 + 4 * q + j] = pack_bf16x2(v0, v1);
     }
   }
