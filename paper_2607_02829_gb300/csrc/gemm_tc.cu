@@ -30,25 +30,33 @@ constexpr int BM = 128, BK = 64;
 constexpr int kThreads = 320;
 constexpr int kEpiThreads = 256;
 
-template <int BN>
+template <int BN, Epi E>
 struct GemmCfg {
-  static constexpr int kStages = BN == 256 ? 4 : 6;
+  // the residual epilogue keeps two 32 x 32 fp32 residual tiles per epilogue
+  // warp in shared memory (64 KB), paid for with a shorter operand ring
+  static constexpr bool kTmaRes = E == Epi::BiasResidual && BN == 128;
+  static constexpr int kStages = kTmaRes ? 4 : (BN == 256 ? 4 : 6);
   static constexpr int kABytes = BM * BK * 2;        // 16 KB
   static constexpr int kBBytes = BN * BK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kTmemCols = 2 * BN;           // two accumulators
   // per epilogue warp: a 32 x 32 fp32 chunk, pitch 33 (conflict-free both ways)
   static constexpr int kStageFloats = 32 * 33;
-  static constexpr size_t kStagingBytes = size_t(kEpiThreads / 32) * kStageFloats * 4;
+  static constexpr int kResTileBytes = 32 * 32 * 4;  // one residual chunk (TMA box)
+  static constexpr size_t kStagingBytes = kTmaRes
+      ? size_t(kEpiThreads / 32) * 2 * kResTileBytes
+      : size_t(kEpiThreads / 32) * kStageFloats * 4;
   static constexpr size_t kSmem =
-      size_t(kStages) * kStageBytes + kStagingBytes + 1024 /*align*/ + 256 /*bars*/;
+      size_t(kStages) * kStageBytes + kStagingBytes + 1024 /*align*/ + 512 /*barriers*/;
 };
 
 struct Smem {
   uint64_t full[8], empty[8], tfull[2], tempty[2], drain;
+  uint64_t res_full[kEpiThreads / 32][2];   // residual tiles landed (per epilogue warp)
   uint32_t tmem_base;
   int abort;
 };
+static_assert(sizeof(Smem) <= 512, "the barrier block must fit its reserve in GemmCfg::kSmem");
 
 // GELU(z) = z * Phi(z) with Phi from the erfc approximation of Abramowitz &
 // Stegun, Handbook of Mathematical Functions, formula 7.1.26 (absolute error
@@ -177,8 +185,8 @@ __device__ __forceinline__ void epilogue32_rows(const EpiArgs& ea, int row0, int
 template <int BN, Epi E>
 __global__ void __launch_bounds__(kThreads, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-               int M, int N, int K, EpiArgs ea) {
-  using C = GemmCfg<BN>;
+               const __grid_constant__ CUtensorMap tmR, int M, int N, int K, EpiArgs ea) {
+  using C = GemmCfg<BN, E>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -198,10 +206,15 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     for (int s = 0; s < C::kStages; ++s) { mbar_init(&sm->full[s], 1); mbar_init(&sm->empty[s], 1); }
     for (int a = 0; a < 2; ++a) { mbar_init(&sm->tfull[a], 1); mbar_init(&sm->tempty[a], kEpiThreads); }
     mbar_init(&sm->drain, 1);
+    for (int w = 0; w < kEpiThreads / 32; ++w) { mbar_init(&sm->res_full[w][0], 1); mbar_init(&sm->res_full[w][1], 1); }
     sm->abort = 0;
     fence_mbar_init();
   }
-  if (warp == 0 && lane == 0) { prefetch_tmap(&tmA); prefetch_tmap(&tmB); }
+  if (warp == 0 && lane == 0) {
+    prefetch_tmap(&tmA);
+    prefetch_tmap(&tmB);
+    if constexpr (C::kTmaRes) prefetch_tmap(&tmR);
+  }
   if (warp == 1) tmem_alloc(&sm->tmem_base, C::kTmemCols);
   tc_fence_before();
   __syncthreads();
@@ -291,6 +304,69 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                                reinterpret_cast<uint32_t*>(staging) + (warp - 2) * C::kStageFloats,
                                lane);
         }
+      } else if constexpr (C::kTmaRes) {
+        // residual tiles by TMA: both chunks of this warp (32 rows x 32 fp32, 128-byte
+        // swizzle) are requested before the accumulator is ready, updated in place
+        // and stored back by TMA
+        static_assert(BN == 128, "the TMA residual epilogue takes two 32-column chunks");
+        unsigned char* rbuf = reinterpret_cast<unsigned char*>(staging) +
+                              size_t(warp - 2) * 2 * C::kResTileBytes;
+        uint64_t* rbar = sm->res_full[warp - 2];
+        if (lane == 0) {
+          bulk_wait_read_all();          // the previous tile's stores left these buffers
+#pragma unroll
+          for (int k = 0; k < 2; ++k) {
+            mbar_arrive_expect_tx(&rbar[k], C::kResTileBytes);
+            tma_load_2d(&tmR, rbuf + k * C::kResTileBytes, &rbar[k], nt * BN + c_begin + 32 * k, row0);
+          }
+        }
+        const uint32_t rph = uint32_t(it) & 1u;
+        bool ok = __all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault));
+        if (ok) {
+          tc_fence_after();
+          const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
+#pragma unroll 1
+          for (int k = 0; k < 2 && ok; ++k) {
+            const int c = c_begin + 32 * k;
+            uint32_t r[32];
+            tmem_ld32(tbase + uint32_t(c), r);
+            tmem_wait_ld();
+            if (!(ok = __all_sync(0xffffffffu, mbar_wait(&rbar[k], rph, abort, ea.fault)))) break;
+            // this thread's row: 16-byte chunk j of the row sits at slot j ^ (row % 8)
+            float4* rowp = reinterpret_cast<float4*>(rbuf + k * C::kResTileBytes + lane * 128);
+            const uint4* bias4 =
+                reinterpret_cast<const uint4*>(static_cast<const bf16*>(ea.bias) + nt * BN + c);
+#pragma unroll
+            for (int jq = 0; jq < 4; ++jq) {
+              const uint4 bq = __ldg(bias4 + jq);
+              const uint32_t bw[4] = {bq.x, bq.y, bq.z, bq.w};
+#pragma unroll
+              for (int h2 = 0; h2 < 2; ++h2) {
+                const int j = 2 * jq + h2;
+                float4 v = rowp[j ^ (lane & 7)];
+                v.x += __uint_as_float(r[4 * j]) + bf16_lo(bw[2 * h2]);
+                v.y += __uint_as_float(r[4 * j + 1]) + bf16_hi(bw[2 * h2]);
+                v.z += __uint_as_float(r[4 * j + 2]) + bf16_lo(bw[2 * h2 + 1]);
+                v.w += __uint_as_float(r[4 * j + 3]) + bf16_hi(bw[2 * h2 + 1]);
+                rowp[j ^ (lane & 7)] = v;
+              }
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0 && row0 < M) {
+              tma_store_2d(&tmR, rbuf + k * C::kResTileBytes, nt * BN + c, row0);
+              bulk_commit_group();
+            }
+          }
+        }
+        if (!ok) {
+          // an aborted pipeline: the residual loads issued above still land first
+          int no_abort = 0;
+          if (lane == 0)
+            for (int k = 0; k < 2; ++k) mbar_wait(&rbar[k], rph, &no_abort, ea.fault);
+          __syncwarp();
+          break;
+        }
       } else {
         // the first chunk's residual loads overlap the wait for the accumulator
         float rv[32];
@@ -310,6 +386,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
       tc_fence_before();
       mbar_arrive(&sm->tempty[acc]);
+    }
+    if constexpr (C::kTmaRes) {
+      if (lane == 0) bulk_wait_all();     // residual stores complete before the CTA exits
     }
   }
   tc_fence_before();
@@ -353,15 +432,39 @@ cudaError_t make_map_2d(CUtensorMap* map, const void* ptr, uint64_t rows, uint64
 
 int g_num_sms = 0;
 
+// 2-D fp32 tensor map over a row-major [rows, cols] matrix, box [32, 32],
+// 128-byte swizzle (the residual stream tiles of the TMA epilogue).
+cudaError_t make_map_f32_32x32(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols) {
+  cudaError_t e = get_encoder();
+  if (e != cudaSuccess) return e;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 4};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(ptr), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 template <int BN, Epi E>
 cudaError_t launch_bn(const void* A, const void* W, int M, int N, int K, const EpiArgs& ea,
                       cudaStream_t s) {
-  using C = GemmCfg<BN>;
-  CUtensorMap ta, tb;
+  using C = GemmCfg<BN, E>;
+  CUtensorMap ta, tb, tr;
   cudaError_t e = make_map_2d(&ta, A, uint64_t(M), uint64_t(K), BM);
   if (e != cudaSuccess) return e;
   e = make_map_2d(&tb, W, uint64_t(N), uint64_t(K), BN);
   if (e != cudaSuccess) return e;
+  if constexpr (C::kTmaRes) {
+    // the update is in place: the residual read and the output are one tensor
+    if (ea.res != ea.out) return cudaErrorInvalidValue;
+    e = make_map_f32_32x32(&tr, ea.out, uint64_t(M), uint64_t(N));
+    if (e != cudaSuccess) return e;
+  } else {
+    tr = tb;    // unused
+  }
   static bool attr_set = false;
   if (!attr_set) {
     e = cudaFuncSetAttribute(gemm_tc_kernel<BN, E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -376,7 +479,7 @@ cudaError_t launch_bn(const void* A, const void* W, int M, int N, int K, const E
   }
   const int tiles = ((M + BM - 1) / BM) * (N / BN);
   const int grid = tiles < g_num_sms ? tiles : g_num_sms;
-  gemm_tc_kernel<BN, E><<<grid, kThreads, C::kSmem, s>>>(ta, tb, M, N, K, ea);
+  gemm_tc_kernel<BN, E><<<grid, kThreads, C::kSmem, s>>>(ta, tb, tr, M, N, K, ea);
   return cudaGetLastError();
 }
 
@@ -386,8 +489,11 @@ cudaError_t launch_epi(Epi epi, const void* A, const void* W, int M, int N, int 
   switch (epi) {
     case Epi::Bias: return launch_bn<BN, Epi::Bias>(A, W, M, N, K, ea, s);
     case Epi::BiasGelu: return launch_bn<BN, Epi::BiasGelu>(A, W, M, N, K, ea, s);
-    case Epi::BiasResidual: return launch_bn<BN, Epi::BiasResidual>(A, W, M, N, K, ea, s);
     case Epi::BiasResidualScatter: return launch_bn<BN, Epi::BiasResidualScatter>(A, W, M, N, K, ea, s);
+    case Epi::BiasResidual:
+      // BN = 128 is the TMA residual epilogue, chosen in launch_gemm_tc
+      if constexpr (BN != 128) return launch_bn<BN, Epi::BiasResidual>(A, W, M, N, K, ea, s);
+      break;
   }
   return cudaErrorInvalidValue;
 }
@@ -397,6 +503,15 @@ cudaError_t launch_epi(Epi epi, const void* A, const void* W, int M, int N, int 
 cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* W, int M, int N, int K,
                            const EpiArgs& ea, cudaStream_t s) {
   if (M < 1 || K % BK != 0 || N % 64 != 0) return cudaErrorInvalidValue;
+  if (epi == Epi::BiasResidual) {
+    // a short mainloop (K <= 2048) cannot hide the fp32 residual traffic behind
+    // the MMAs: 128-column tiles with the TMA residual epilogue; a long one keeps
+    // 256-column tiles and the register epilogue
+    if (N % 128 == 0 && (K <= 2048 || N % 256 != 0))
+      return launch_bn<128, Epi::BiasResidual>(A, W, M, N, K, ea, s);
+    if (N % 256 == 0) return launch_epi<256>(epi, A, W, M, N, K, ea, s);
+    return launch_epi<64>(epi, A, W, M, N, K, ea, s);
+  }
   if (N % 256 == 0) return launch_epi<256>(epi, A, W, M, N, K, ea, s);
   if (N % 128 == 0) return launch_epi<128>(epi, A, W, M, N, K, ea, s);
   return launch_epi<64>(epi, A, W, M, N, K, ea, s);
