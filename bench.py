@@ -125,6 +125,33 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def rank_inputs(wl, rank):
+    """One replica's inputs: its own batch (input seed offset by the rank) and the
+    model's weights, the same on every rank.  CPU tensors in the storage dtype."""
+    from paper_2607_02829_gb300 import synth
+    xw = wl.with_(seed_index=wl.seed_index + 100 * rank) if rank else wl
+    x = synth.to_storage(synth.make_tokens(xw), wl.dtype)
+    ws = [{k: synth.to_storage(v, wl.dtype) for k, v in blk.items()}
+          for blk in synth.make_weights(wl)]
+    return x, ws
+
+
+def max_over_ranks(value, world, device):
+    """The largest value over all ranks (every rank gets it); the value itself at N=1."""
+    if world == 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(tokens_per_rank, world, ms_slowest):
+    """Whole-job throughput: every replica's tokens over the slowest rank's time."""
+    return tokens_per_rank * world / (ms_slowest * 1e-3)
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -138,8 +165,7 @@ def run_ours(args, rank, world, local_rank):
                         selector=wl.selector)
     enc = b.Encoder(cfg, max_keep_ratio=wl.keep_ratio)
     # each rank: its own batch (seeded by rank), shared weights
-    x_cpu, w_cpu = synth.make_inputs(wl.with_(seed_index=wl.seed_index + 100 * rank)
-                                     if rank else wl)
+    x_cpu, w_cpu = rank_inputs(wl, rank)
     x = x_cpu.to(dev)
     wd = [{k: v.to(dev) for k, v in blk.items()} for blk in w_cpu]
     warr = b.weights_array(wd)
@@ -178,10 +204,7 @@ def run_ours(args, rank, world, local_rank):
     wall = time.perf_counter() - t0
     clk = clocks.stop()
     ms = sum(a.elapsed_time(z) for a, z in ev) / args.steps
-    ms_t = torch.tensor([ms], device=dev)
-    if world > 1:
-        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
-    ms = float(ms_t.item())
+    ms = max_over_ranks(ms, world, dev)
 
     # ---- per-kernel trace over K more steps (same launches, events around each)
     b.sr_trace_enable(enc.handle, True)
@@ -239,10 +262,7 @@ def run_ours(args, rank, world, local_rank):
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / args.steps
-    e2e_t = torch.tensor([e2e_ms], device=dev)
-    if world > 1:
-        dist.all_reduce(e2e_t, op=dist.ReduceOp.MAX)
-    e2e_ms = float(e2e_t.item())
+    e2e_ms = max_over_ranks(e2e_ms, world, dev)
     enc.close()
     return wl, K, ms, wall, clk, trace, e2e_ms, bytes_io, segment
 
@@ -362,7 +382,7 @@ def main():
                                                                        local_rank)
     peaks = _peaks()
     tokens = wl.B * wl.L * world
-    value = tokens / (ms * 1e-3)
+    value = job_tokens_per_s(wl.B * wl.L, world, ms)
     roof, detail = roofline(trace, peaks, args.steps, wl.name, fp32_alu=wl.dtype == "f32")
     launches = sum(v["launches"] for v in trace.values())
     gs = {}
@@ -389,7 +409,7 @@ def main():
                                      "sparse blocks")
                            if segment and wl.dtype == "bf16" else segment),
         "kernels": detail,
-        "e2e": {"value": tokens / (e2e_ms * 1e-3), "unit": "tokens/s",
+        "e2e": {"value": job_tokens_per_s(wl.B * wl.L, world, e2e_ms), "unit": "tokens/s",
                 "h2d_bytes_per_step": bytes_io, "d2h_bytes_per_step": bytes_io},
         "gpu_launches": int(launches),
         "wall_s_timed_region": wall,
