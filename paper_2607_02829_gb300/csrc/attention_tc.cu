@@ -16,8 +16,12 @@
 //               issued as soon as softmax t has read the current one;
 //   warps 4-7   softmax of tile 0, warps 8-11 softmax of tile 1: one query row
 //               per thread.  Each reads its S row from TMEM, updates the
-//               running max and sum, and writes P = 2^(s*c - m*c) as bf16
-//               pairs into tensor memory, where the P V MMA reads its A operand.
+//               running max and sum, computes P = 2^(s*c - m*c) as bf16 pairs
+//               in registers and, once the previous P V has read the tile's P
+//               columns, writes them to tensor memory, where the P V MMA reads
+//               its A operand.
+// setmaxnreg moves registers from the load / MMA warpgroup (56 per thread) to
+// the softmax warpgroups (224), which hold a whole S row and P row at once.
 // The running max is only raised when it grows by more than 2^8 (in the exp2
 // domain); then the thread rescales its O row in TMEM first.  P, O and the sum
 // always use the same max, so the result is exact up to rounding.
@@ -108,93 +112,100 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
   const uint32_t tmem = sm->tmem_base;
   volatile int* abort = &sm->abort;
 
-  if (warp == 0 || warp == 3) {
-    // ------------------------------------------------------------- TMA loads
-    // warp 0: the Q tiles, then K_j; warp 3: V_j
-    if (lane == 0) {
-      const bool is_k = warp == 0;
-      if (is_k) {
-        mbar_arrive_expect_tx(&sm->q_full, kQTiles * kTileBytes);
-        for (int t = 0; t < kQTiles; ++t)
-          tma_load_3d(&tm, sQ + t * kTileBytes, &sm->q_full, h * kDh, q0 + t * kQTile, b);
-      }
-      uint64_t* full = is_k ? sm->k_full : sm->v_full;
-      uint64_t* empty = is_k ? sm->k_empty : sm->v_empty;
-      unsigned char* ring = is_k ? sK : sV;
-      const int col = (is_k ? D : 2 * D) + h * kDh;
-      uint32_t issued = 0, par = 0;   // stages holding a load; parity of its phase
-      int st = 0;
-      uint32_t ph = 0;
-      for (int j = 0; j < nkv; ++j) {
-        // the stage is free once both tiles' MMAs of key tile j - kStages have read it
-        if (!mbar_wait(&empty[st], ph ^ 1, abort, fault)) break;
-        mbar_arrive_expect_tx(&full[st], kTileBytes);
-        tma_load_3d(&tm, ring + st * kTileBytes, &full[st], col, j * kKV, b);
-        issued |= 1u << st;
-        par = (par & ~(1u << st)) | (ph << st);
-        if (++st == kStages) { st = 0; ph ^= 1; }
-      }
-      // every issued load lands before the CTA may exit
-      int no_abort = 0;
-      if (is_k) mbar_wait(&sm->q_full, 0, &no_abort, fault);
-      for (int s = 0; s < kStages; ++s)
-        if (issued & (1u << s)) mbar_wait(&full[s], (par >> s) & 1u, &no_abort, fault);
-    }
-  } else if (warp == 1 || warp == 2) {
-    // ------------------------------------------------------------- MMA issue
-    // warp 1 issues tile 0's MMAs, warp 2 tile 1's, each in its own order
-    if (lane == 0) {
-      const int t = warp - 1;
-      constexpr uint32_t idesc_s = idesc_bf16(kQTile, kKV);                 // K-major A, B
-      constexpr uint32_t idesc_o = idesc_bf16(kQTile, kDh, false, true);   // V is MN-major
-      const uint32_t dS = tmem + kColS + uint32_t(t * kKV);
-      const uint32_t dO = tmem + kColO + uint32_t(t * kDh);
-      const uint32_t qa = smem_u32(sQ + t * kTileBytes);
-      auto issue_s = [&](int st) {
-        const uint32_t ka = smem_u32(sK + st * kTileBytes);
-#pragma unroll
-        for (int k = 0; k < kDh / 16; ++k)
-          mma_bf16(dS, sw128_desc(qa + 32 * k), sw128_desc(ka + 32 * k), idesc_s, k > 0 ? 1u : 0u);
-        mma_commit(&sm->s_full[t]);
-        mma_commit(&sm->k_empty[st]);
-      };
-      bool ok = mbar_wait(&sm->q_full, 0, abort, fault);
-      if (ok) ok = mbar_wait(&sm->k_full[0], 0, abort, fault);
-      if (ok) {
-        tc_fence_after();
-        issue_s(0);
-      }
-      const uint32_t aP = tmem + kColP + uint32_t(t * (kKV / 2));
-      int vs = 0;                 // stage of V_j
-      uint32_t vph = 0;
-      for (int j = 0; j < nkv && ok; ++j) {
-        // S for the next key tile as soon as the softmax has read this one
-        if (j + 1 < nkv) {
-          const int st = vs + 1 == kStages ? 0 : vs + 1;
-          const uint32_t sph = vs + 1 == kStages ? vph ^ 1 : vph;
-          if (!(ok = mbar_wait(&sm->k_full[st], sph, abort, fault))) break;
-          if (!(ok = mbar_wait(&sm->s_free[t], j & 1, abort, fault))) break;
-          tc_fence_after();
-          issue_s(st);
+  if (warp < 4) {
+    // registers: 56 per thread for the load / MMA warpgroup, 224 for the two
+    // softmax warpgroups; 128 * 56 + 256 * 224 = 384 * 168, the launch's total
+    // (the launcher checks that the kernel was built with 168)
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 56;\n" ::: "memory");
+    if (warp == 0 || warp == 3) {
+      // ------------------------------------------------------------- TMA loads
+      // warp 0: the Q tiles, then K_j; warp 3: V_j
+      if (lane == 0) {
+        const bool is_k = warp == 0;
+        if (is_k) {
+          mbar_arrive_expect_tx(&sm->q_full, kQTiles * kTileBytes);
+          for (int t = 0; t < kQTiles; ++t)
+            tma_load_3d(&tm, sQ + t * kTileBytes, &sm->q_full, h * kDh, q0 + t * kQTile, b);
         }
-        // O^t += P^t_j V_j with P read from tensor memory (64 columns of bf16 pairs)
-        if (!(ok = mbar_wait(&sm->v_full[vs], vph, abort, fault))) break;
-        if (!(ok = mbar_wait(&sm->p_full[t], j & 1, abort, fault))) break;
-        tc_fence_after();
-        const uint32_t va = smem_u32(sV + vs * kTileBytes);
-#pragma unroll
-        for (int k = 0; k < kKV / 16; ++k)
-          mma_bf16_ts(dO, aP + uint32_t(k * 8), sw128_desc_mn(va + k * 2048), idesc_o,
-                      (j | k) != 0 ? 1u : 0u);
-        mma_commit(&sm->pv_done[t]);
-        mma_commit(&sm->v_empty[vs]);
-        if (++vs == kStages) { vs = 0; vph ^= 1; }
+        uint64_t* full = is_k ? sm->k_full : sm->v_full;
+        uint64_t* empty = is_k ? sm->k_empty : sm->v_empty;
+        unsigned char* ring = is_k ? sK : sV;
+        const int col = (is_k ? D : 2 * D) + h * kDh;
+        uint32_t issued = 0, par = 0;   // stages holding a load; parity of its phase
+        int st = 0;
+        uint32_t ph = 0;
+        for (int j = 0; j < nkv; ++j) {
+          // the stage is free once both tiles' MMAs of key tile j - kStages have read it
+          if (!mbar_wait(&empty[st], ph ^ 1, abort, fault)) break;
+          mbar_arrive_expect_tx(&full[st], kTileBytes);
+          tma_load_3d(&tm, ring + st * kTileBytes, &full[st], col, j * kKV, b);
+          issued |= 1u << st;
+          par = (par & ~(1u << st)) | (ph << st);
+          if (++st == kStages) { st = 0; ph ^= 1; }
+        }
+        // every issued load lands before the CTA may exit
+        int no_abort = 0;
+        if (is_k) mbar_wait(&sm->q_full, 0, &no_abort, fault);
+        for (int s = 0; s < kStages; ++s)
+          if (issued & (1u << s)) mbar_wait(&full[s], (par >> s) & 1u, &no_abort, fault);
       }
-      int no_abort = 0;
-      mma_commit(&sm->drain[t]);
-      mbar_wait(&sm->drain[t], 0, &no_abort, fault);
+    } else if (warp == 1 || warp == 2) {
+      // ------------------------------------------------------------- MMA issue
+      // warp 1 issues tile 0's MMAs, warp 2 tile 1's, each in its own order
+      if (lane == 0) {
+        const int t = warp - 1;
+        constexpr uint32_t idesc_s = idesc_bf16(kQTile, kKV);                 // K-major A, B
+        constexpr uint32_t idesc_o = idesc_bf16(kQTile, kDh, false, true);   // V is MN-major
+        const uint32_t dS = tmem + kColS + uint32_t(t * kKV);
+        const uint32_t dO = tmem + kColO + uint32_t(t * kDh);
+        const uint32_t qa = smem_u32(sQ + t * kTileBytes);
+        auto issue_s = [&](int st) {
+          const uint32_t ka = smem_u32(sK + st * kTileBytes);
+  #pragma unroll
+          for (int k = 0; k < kDh / 16; ++k)
+            mma_bf16(dS, sw128_desc(qa + 32 * k), sw128_desc(ka + 32 * k), idesc_s, k > 0 ? 1u : 0u);
+          mma_commit(&sm->s_full[t]);
+          mma_commit(&sm->k_empty[st]);
+        };
+        bool ok = mbar_wait(&sm->q_full, 0, abort, fault);
+        if (ok) ok = mbar_wait(&sm->k_full[0], 0, abort, fault);
+        if (ok) {
+          tc_fence_after();
+          issue_s(0);
+        }
+        const uint32_t aP = tmem + kColP + uint32_t(t * (kKV / 2));
+        int vs = 0;                 // stage of V_j
+        uint32_t vph = 0;
+        for (int j = 0; j < nkv && ok; ++j) {
+          // S for the next key tile as soon as the softmax has read this one
+          if (j + 1 < nkv) {
+            const int st = vs + 1 == kStages ? 0 : vs + 1;
+            const uint32_t sph = vs + 1 == kStages ? vph ^ 1 : vph;
+            if (!(ok = mbar_wait(&sm->k_full[st], sph, abort, fault))) break;
+            if (!(ok = mbar_wait(&sm->s_free[t], j & 1, abort, fault))) break;
+            tc_fence_after();
+            issue_s(st);
+          }
+          // O^t += P^t_j V_j with P read from tensor memory (64 columns of bf16 pairs)
+          if (!(ok = mbar_wait(&sm->v_full[vs], vph, abort, fault))) break;
+          if (!(ok = mbar_wait(&sm->p_full[t], j & 1, abort, fault))) break;
+          tc_fence_after();
+          const uint32_t va = smem_u32(sV + vs * kTileBytes);
+  #pragma unroll
+          for (int k = 0; k < kKV / 16; ++k)
+            mma_bf16_ts(dO, aP + uint32_t(k * 8), sw128_desc_mn(va + k * 2048), idesc_o,
+                        (j | k) != 0 ? 1u : 0u);
+          mma_commit(&sm->pv_done[t]);
+          mma_commit(&sm->v_empty[vs]);
+          if (++vs == kStages) { vs = 0; vph ^= 1; }
+        }
+        int no_abort = 0;
+        mma_commit(&sm->drain[t]);
+        mbar_wait(&sm->drain[t], 0, &no_abort, fault);
+      }
     }
   } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 224;\n" ::: "memory");
     // ------------------------------------------------------------- softmax
     const int t = (warp - 4) >> 2;                 // query tile of this warpgroup
     const int quarter = warp & 3;                  // TMEM lane quarter
@@ -250,20 +261,15 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
         l_run *= alpha;
         rescale = true;
       }
-      // P and O of this tile are free once the previous P V has completed
-      if (j >= 1) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (j - 1) & 1, abort, fault));
-        if (!ok) break;
-        tc_fence_after();
-      }
-      // P = 2^(s c - m c) as bf16 pairs into tensor memory: key 2i and 2i+1 of
-      // this row share column i of the tile's P region (the A operand of P V)
+      // P = 2^(s c - m c) as bf16 pairs, held in registers until the previous
+      // P V has released the tile's P columns: key 2i and 2i+1 of this row share
+      // column i of the tile's P region (the A operand of P V)
       const float mc = m_run * c;
       const uint64_t nmc2 = pk2(-mc, -mc);
       uint64_t ls2[2] = {pk2(0.f, 0.f), pk2(0.f, 0.f)};
+      uint32_t w[kKV / 64][32];
 #pragma unroll
       for (int cc = 0; cc < kKV / 32; ++cc) {
-        uint32_t w[16];
 #pragma unroll
         for (int q = 0; q < 16; ++q) {
           const int i0 = 32 * cc + 2 * q;
@@ -272,11 +278,12 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
                                     c2, nmc2);
           float a0, a1;
           up2(arg, a0, a1);
-          const float p0 = ex2(a0), p1 = ex2(a1);
-          ls2[q & 1] = add2(ls2[q & 1], pk2(p0, p1));
-          w[q] = pack_bf16x2(p0, p1);
+          const uint64_t p2 = pk2(ex2(a0), ex2(a1));
+          ls2[q & 1] = add2(ls2[q & 1], p2);
+          float p0, p1;
+          up2(p2, p0, p1);
+          w[cc / 2][(cc % 2) * 16 + q] = pack_bf16x2(p0, p1);
         }
-        tmem_st16(tP + uint32_t(cc * 16), w);
       }
       {
         float l0, l1, l2, l3;
@@ -284,6 +291,14 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
         up2(ls2[1], l2, l3);
         l_run += (l0 + l1) + (l2 + l3);
       }
+      // P and O of this tile are free once the previous P V has completed
+      if (j >= 1) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (j - 1) & 1, abort, fault));
+        if (!ok) break;
+        tc_fence_after();
+      }
+#pragma unroll
+      for (int hh = 0; hh < kKV / 64; ++hh) tmem_st32(tP + uint32_t(hh * 32), w[hh]);
       // a raised max rescales O, which holds every earlier P V product
       if (__any_sync(0xffffffffu, rescale)) {
         uint32_t o[32];
@@ -365,6 +380,10 @@ cudaError_t launch_attention_tc(const void* qkv, void* out, int B, int T, int he
   if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
   static bool attr_set = false;
   if (!attr_set) {
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, attention_tc_kernel);
+    if (e != cudaSuccess) return e;
+    if (fa.numRegs < 168) return cudaErrorInvalidConfiguration;   // the register split needs 168
     e = cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              int(kSmemBytes));
     if (e != cudaSuccess) return e;
