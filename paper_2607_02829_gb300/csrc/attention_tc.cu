@@ -6,14 +6,17 @@
 //
 // One CTA owns 256 query rows of one (sample, head) as two 128-row tiles that
 // share every K/V tile, 384 threads:
-//   warps 0, 3  TMA: the two Q tiles once, then K_j (warp 0) and V_j (warp 3),
-//               128 keys x 64, into two 3-stage rings (3-D tensor map over
-//               [B, T, 3D], zero fill past T); a K stage frees as soon as both
-//               tiles' S MMAs that read it finish, a V stage when the P V MMAs do;
-//   warps 1, 2  tcgen05.mma for tile 0 and tile 1, each thread in its own order:
-//               S^t = Q^t K_j^T (128 x 128, fp32 in TMEM), O^t += P^t V_j
-//               (128 x 64, accumulated in TMEM, P from TMEM); the next S^t is
-//               issued as soon as softmax t has read the current one;
+//   warp 0      TMA: the two Q tiles once, then K_j and V_j, 128 keys x 64, into
+//               two 3-stage rings (3-D tensor map over [B, T, 3D], zero fill
+//               past T); a K stage frees as soon as both tiles' S MMAs that read
+//               it finish, a V stage when both tiles' P V MMAs do;
+//   warp 1      issues S^t = Q^t K_j^T (128 x 128, fp32 in TMEM) for both tiles,
+//               each as soon as softmax t has read the previous one;
+//   warps 2, 3  issue O^t += P^t V_j for tile 0 and tile 1 (128 x 64,
+//               accumulated in TMEM, P read from TMEM).  One thread issues a
+//               tcgen05.mma only about every 120 cycles whatever its shape, and
+//               an N = 64 MMA is 32 cycles of work, so the P V MMAs of each tile
+//               get their own issuing thread;
 //   warps 4-7   softmax of tile 0, warps 8-11 softmax of tile 1: one query row
 //               per thread.  Each reads its S row from TMEM, updates the
 //               running max and sum, computes P = 2^(s*c - m*c) as bf16 pairs
@@ -53,13 +56,14 @@ struct AttSmem {
   uint64_t q_full;
   uint64_t k_full[kStages], k_empty[kStages], v_full[kStages], v_empty[kStages];
   uint64_t s_full[kQTiles], s_free[kQTiles], p_full[kQTiles], pv_done[kQTiles];
-  uint64_t drain[kQTiles];
+  uint64_t drain[1 + kQTiles];      // the S issuer, then each P V issuer
   uint32_t tmem_base;
   int abort;
 };
 
 constexpr size_t kSmemBytes = 1024 /*align*/ + size_t(kQTiles) * kTileBytes +
                               size_t(kStages) * 2 * kTileBytes + 256;
+static_assert(sizeof(AttSmem) <= 256, "barrier block outgrew its reserve");
 
 __device__ __forceinline__ float max3(float a, float b, float c) {
   float d;
@@ -90,8 +94,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
   if (threadIdx.x == 0) {
     mbar_init(&sm->q_full, 1);
     for (int s = 0; s < kStages; ++s) {
-      // a stage is released by both MMA threads
-      mbar_init(&sm->k_full[s], 1); mbar_init(&sm->k_empty[s], kQTiles);
+      // a K stage is released by the S issuer, a V stage by both P V issuers
+      mbar_init(&sm->k_full[s], 1); mbar_init(&sm->k_empty[s], 1);
       mbar_init(&sm->v_full[s], 1); mbar_init(&sm->v_empty[s], kQTiles);
     }
     for (int t = 0; t < kQTiles; ++t) {
@@ -99,8 +103,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
       mbar_init(&sm->s_free[t], kQTile);
       mbar_init(&sm->p_full[t], kQTile);
       mbar_init(&sm->pv_done[t], 1);
-      mbar_init(&sm->drain[t], 1);
     }
+    for (int d = 0; d < 1 + kQTiles; ++d) mbar_init(&sm->drain[d], 1);
     sm->abort = 0;
     fence_mbar_init();
   }
@@ -117,91 +121,100 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
     // softmax warpgroups; 128 * 56 + 256 * 224 = 384 * 168, the launch's total
     // (the launcher checks that the kernel was built with 168)
     asm volatile("setmaxnreg.dec.sync.aligned.u32 56;\n" ::: "memory");
-    if (warp == 0 || warp == 3) {
+    if (warp == 0) {
       // ------------------------------------------------------------- TMA loads
-      // warp 0: the Q tiles, then K_j; warp 3: V_j
+      // the two Q tiles once, then K_j and V_j into their rings
       if (lane == 0) {
-        const bool is_k = warp == 0;
-        if (is_k) {
-          mbar_arrive_expect_tx(&sm->q_full, kQTiles * kTileBytes);
-          for (int t = 0; t < kQTiles; ++t)
-            tma_load_3d(&tm, sQ + t * kTileBytes, &sm->q_full, h * kDh, q0 + t * kQTile, b);
-        }
-        uint64_t* full = is_k ? sm->k_full : sm->v_full;
-        uint64_t* empty = is_k ? sm->k_empty : sm->v_empty;
-        unsigned char* ring = is_k ? sK : sV;
-        const int col = (is_k ? D : 2 * D) + h * kDh;
-        uint32_t issued = 0, par = 0;   // stages holding a load; parity of its phase
+        mbar_arrive_expect_tx(&sm->q_full, kQTiles * kTileBytes);
+        for (int t = 0; t < kQTiles; ++t)
+          tma_load_3d(&tm, sQ + t * kTileBytes, &sm->q_full, h * kDh, q0 + t * kQTile, b);
+        const int kcol = D + h * kDh, vcol = 2 * D + h * kDh;
+        // stages holding a load, and the parity of the phase each last used
+        uint32_t kissued = 0, vissued = 0, kpar = 0, vpar = 0;
         int st = 0;
         uint32_t ph = 0;
         for (int j = 0; j < nkv; ++j) {
-          // the stage is free once both tiles' MMAs of key tile j - kStages have read it
-          if (!mbar_wait(&empty[st], ph ^ 1, abort, fault)) break;
-          mbar_arrive_expect_tx(&full[st], kTileBytes);
-          tma_load_3d(&tm, ring + st * kTileBytes, &full[st], col, j * kKV, b);
-          issued |= 1u << st;
-          par = (par & ~(1u << st)) | (ph << st);
+          // a K stage frees once both tiles' S MMAs of key tile j - kStages are done
+          if (!mbar_wait(&sm->k_empty[st], ph ^ 1, abort, fault)) break;
+          mbar_arrive_expect_tx(&sm->k_full[st], kTileBytes);
+          tma_load_3d(&tm, sK + st * kTileBytes, &sm->k_full[st], kcol, j * kKV, b);
+          kissued |= 1u << st;
+          kpar = (kpar & ~(1u << st)) | (ph << st);
+          // a V stage once both tiles' P V MMAs of that key tile are
+          if (!mbar_wait(&sm->v_empty[st], ph ^ 1, abort, fault)) break;
+          mbar_arrive_expect_tx(&sm->v_full[st], kTileBytes);
+          tma_load_3d(&tm, sV + st * kTileBytes, &sm->v_full[st], vcol, j * kKV, b);
+          vissued |= 1u << st;
+          vpar = (vpar & ~(1u << st)) | (ph << st);
           if (++st == kStages) { st = 0; ph ^= 1; }
         }
         // every issued load lands before the CTA may exit
         int no_abort = 0;
-        if (is_k) mbar_wait(&sm->q_full, 0, &no_abort, fault);
-        for (int s = 0; s < kStages; ++s)
-          if (issued & (1u << s)) mbar_wait(&full[s], (par >> s) & 1u, &no_abort, fault);
-      }
-    } else if (warp == 1 || warp == 2) {
-      // ------------------------------------------------------------- MMA issue
-      // warp 1 issues tile 0's MMAs, warp 2 tile 1's, each in its own order
-      if (lane == 0) {
-        const int t = warp - 1;
-        constexpr uint32_t idesc_s = idesc_bf16(kQTile, kKV);                 // K-major A, B
-        constexpr uint32_t idesc_o = idesc_bf16(kQTile, kDh, false, true);   // V is MN-major
-        const uint32_t dS = tmem + kColS + uint32_t(t * kKV);
-        const uint32_t dO = tmem + kColO + uint32_t(t * kDh);
-        const uint32_t qa = smem_u32(sQ + t * kTileBytes);
-        auto issue_s = [&](int st) {
-          const uint32_t ka = smem_u32(sK + st * kTileBytes);
-  #pragma unroll
-          for (int k = 0; k < kDh / 16; ++k)
-            mma_bf16(dS, sw128_desc(qa + 32 * k), sw128_desc(ka + 32 * k), idesc_s, k > 0 ? 1u : 0u);
-          mma_commit(&sm->s_full[t]);
-          mma_commit(&sm->k_empty[st]);
-        };
-        bool ok = mbar_wait(&sm->q_full, 0, abort, fault);
-        if (ok) ok = mbar_wait(&sm->k_full[0], 0, abort, fault);
-        if (ok) {
-          tc_fence_after();
-          issue_s(0);
+        mbar_wait(&sm->q_full, 0, &no_abort, fault);
+        for (int s = 0; s < kStages; ++s) {
+          if (kissued & (1u << s)) mbar_wait(&sm->k_full[s], (kpar >> s) & 1u, &no_abort, fault);
+          if (vissued & (1u << s)) mbar_wait(&sm->v_full[s], (vpar >> s) & 1u, &no_abort, fault);
         }
-        const uint32_t aP = tmem + kColP + uint32_t(t * (kKV / 2));
-        int vs = 0;                 // stage of V_j
-        uint32_t vph = 0;
+      }
+    } else if (warp == 1) {
+      // ------------------------------------------------------------- S MMAs
+      // S^t = Q^t K_j^T for both tiles, each once softmax t has read S^t of key
+      // tile j - 1
+      if (lane == 0) {
+        constexpr uint32_t idesc_s = idesc_bf16(kQTile, kKV);                 // K-major A, B
+        bool ok = mbar_wait(&sm->q_full, 0, abort, fault);
+        int st = 0;
+        uint32_t ph = 0;
         for (int j = 0; j < nkv && ok; ++j) {
-          // S for the next key tile as soon as the softmax has read this one
-          if (j + 1 < nkv) {
-            const int st = vs + 1 == kStages ? 0 : vs + 1;
-            const uint32_t sph = vs + 1 == kStages ? vph ^ 1 : vph;
-            if (!(ok = mbar_wait(&sm->k_full[st], sph, abort, fault))) break;
-            if (!(ok = mbar_wait(&sm->s_free[t], j & 1, abort, fault))) break;
+          if (!(ok = mbar_wait(&sm->k_full[st], ph, abort, fault))) break;
+          const uint32_t ka = smem_u32(sK + st * kTileBytes);
+          for (int t = 0; t < kQTiles && ok; ++t) {
+            if (j > 0 && !(ok = mbar_wait(&sm->s_free[t], (j - 1) & 1, abort, fault))) break;
             tc_fence_after();
-            issue_s(st);
+            const uint32_t qa = smem_u32(sQ + t * kTileBytes);
+            const uint32_t dS = tmem + kColS + uint32_t(t * kKV);
+#pragma unroll
+            for (int k = 0; k < kDh / 16; ++k)
+              mma_bf16(dS, sw128_desc(qa + 32 * k), sw128_desc(ka + 32 * k), idesc_s,
+                       k > 0 ? 1u : 0u);
+            mma_commit(&sm->s_full[t]);
           }
-          // O^t += P^t_j V_j with P read from tensor memory (64 columns of bf16 pairs)
-          if (!(ok = mbar_wait(&sm->v_full[vs], vph, abort, fault))) break;
+          if (!ok) break;
+          mma_commit(&sm->k_empty[st]);
+          if (++st == kStages) { st = 0; ph ^= 1; }
+        }
+        int no_abort = 0;
+        mma_commit(&sm->drain[0]);
+        mbar_wait(&sm->drain[0], 0, &no_abort, fault);
+      }
+    } else {
+      // ------------------------------------------------------------- P V MMAs
+      // warp 2 for tile 0, warp 3 for tile 1: O^t += P^t_j V_j (128 x 64,
+      // accumulated in TMEM), P read from TMEM (64 columns of bf16 pairs)
+      if (lane == 0) {
+        const int t = warp - 2;
+        constexpr uint32_t idesc_o = idesc_bf16(kQTile, kDh, false, true);   // V is MN-major
+        const uint32_t dO = tmem + kColO + uint32_t(t * kDh);
+        const uint32_t aP = tmem + kColP + uint32_t(t * (kKV / 2));
+        bool ok = true;
+        int st = 0;
+        uint32_t ph = 0;
+        for (int j = 0; j < nkv && ok; ++j) {
+          if (!(ok = mbar_wait(&sm->v_full[st], ph, abort, fault))) break;
           if (!(ok = mbar_wait(&sm->p_full[t], j & 1, abort, fault))) break;
           tc_fence_after();
-          const uint32_t va = smem_u32(sV + vs * kTileBytes);
-  #pragma unroll
+          const uint32_t va = smem_u32(sV + st * kTileBytes);
+#pragma unroll
           for (int k = 0; k < kKV / 16; ++k)
             mma_bf16_ts(dO, aP + uint32_t(k * 8), sw128_desc_mn(va + k * 2048), idesc_o,
                         (j | k) != 0 ? 1u : 0u);
           mma_commit(&sm->pv_done[t]);
-          mma_commit(&sm->v_empty[vs]);
-          if (++vs == kStages) { vs = 0; vph ^= 1; }
+          mma_commit(&sm->v_empty[st]);
+          if (++st == kStages) { st = 0; ph ^= 1; }
         }
         int no_abort = 0;
-        mma_commit(&sm->drain[t]);
-        mbar_wait(&sm->drain[t], 0, &no_abort, fault);
+        mma_commit(&sm->drain[1 + t]);
+        mbar_wait(&sm->drain[1 + t], 0, &no_abort, fault);
       }
     }
   } else {
