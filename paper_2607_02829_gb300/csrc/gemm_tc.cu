@@ -35,6 +35,10 @@ struct GemmCfg {
   // the residual epilogue keeps two 32 x 32 fp32 residual tiles per epilogue
   // warp in shared memory (64 KB), paid for with a shorter operand ring
   static constexpr bool kTmaRes = E == Epi::BiasResidual && BN == 128;
+  // bf16 outputs of tiles at least 128 columns wide leave through TMA stores
+  // from a 128-byte-swizzled 32 x 64 tile per epilogue warp (4 KB)
+  static constexpr bool kTmaOut = (E == Epi::Bias || E == Epi::BiasGelu) && BN >= 128;
+  static constexpr int kOutTileBytes = 32 * 128;
   static constexpr int kStages = kTmaRes ? 4 : (BN == 256 ? 4 : 6);
   static constexpr int kABytes = BM * BK * 2;        // 16 KB
   static constexpr int kBBytes = BN * BK * 2;
@@ -45,7 +49,8 @@ struct GemmCfg {
   static constexpr int kResTileBytes = 32 * 32 * 4;  // one residual chunk (TMA box)
   static constexpr size_t kStagingBytes = kTmaRes
       ? size_t(kEpiThreads / 32) * 2 * kResTileBytes
-      : size_t(kEpiThreads / 32) * kStageFloats * 4;
+      : kTmaOut ? size_t(kEpiThreads / 32) * kOutTileBytes
+                : size_t(kEpiThreads / 32) * kStageFloats * 4;
   static constexpr size_t kSmem =
       size_t(kStages) * kStageBytes + kStagingBytes + 1024 /*align*/ + 512 /*barriers*/;
 };
@@ -85,6 +90,27 @@ __device__ __forceinline__ void gelu2_as7126(float& z0, float& z1) {
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Bias (and GELU) on this thread's row of 64 accumulators (columns n..n+63),
+// packed into 32 bf16 pairs.
+template <Epi E>
+__device__ __forceinline__ void bias_act_pack64(const EpiArgs& ea, int n, const uint32_t (&acc)[2][32],
+                                                uint32_t (&wv)[32]) {
+  const uint4* bias4 = reinterpret_cast<const uint4*>(static_cast<const bf16*>(ea.bias) + n);
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const uint4 bq = __ldg(bias4 + q);
+    const uint32_t bw[4] = {bq.x, bq.y, bq.z, bq.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int c0 = 8 * q + 2 * j;
+      float v0 = __uint_as_float(acc[c0 / 32][c0 % 32]) + bf16_lo(bw[j]);
+      float v1 = __uint_as_float(acc[(c0 + 1) / 32][(c0 + 1) % 32]) + bf16_hi(bw[j]);
+      if constexpr (E == Epi::BiasGelu) gelu2_as7126(v0, v1);
+      wv[4 * q + j] = pack_bf16x2(v0, v1);
+    }
+  }
+}
 
 // bf16 epilogues (bias; bias + GELU) over W = 64 or 32 consecutive columns
 // n..n+W-1 of the warp's 32 rows row0..row0+31: each thread biases (and GELUs)
@@ -213,7 +239,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   if (warp == 0 && lane == 0) {
     prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
-    if constexpr (C::kTmaRes) prefetch_tmap(&tmR);
+    if constexpr (C::kTmaRes || C::kTmaOut) prefetch_tmap(&tmR);
   }
   if (warp == 1) tmem_alloc(&sm->tmem_base, C::kTmemCols);
   tc_fence_before();
@@ -290,7 +316,37 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       const uint32_t aphase = (it >> 1) & 1;
       const int row0 = mt * BM + q * 32;
       const int c_begin = half * (BN / 2), c_end = (half + 1) * (BN / 2);
-      if constexpr (E == Epi::Bias || E == Epi::BiasGelu) {
+      if constexpr (C::kTmaOut) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault))) break;
+        tc_fence_after();
+        const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
+        unsigned char* obuf = reinterpret_cast<unsigned char*>(staging) +
+                              size_t(warp - 2) * C::kOutTileBytes;
+#pragma unroll 1
+        for (int c = c_begin; c < c_end; c += 64) {
+          uint32_t r[2][32];
+          tmem_ld32(tbase + uint32_t(c), r[0]);
+          tmem_ld32(tbase + uint32_t(c + 32), r[1]);
+          tmem_wait_ld();
+          uint32_t wv[32];
+          bias_act_pack64<E>(ea, nt * BN + c, r, wv);
+          // the previous store from this buffer has read it before it is rewritten
+          if (lane == 0) bulk_wait_read_all();
+          __syncwarp();
+          // this thread's row: 16-byte chunk j of the row sits at slot j ^ (row % 8)
+          uint4* rowp = reinterpret_cast<uint4*>(obuf + lane * 128);
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            rowp[j ^ (lane & 7)] = make_uint4(wv[4 * j], wv[4 * j + 1], wv[4 * j + 2], wv[4 * j + 3]);
+          fence_proxy_async_smem();
+          __syncwarp();
+          // rows past M are clipped by the tensor map
+          if (lane == 0 && row0 < M) {
+            tma_store_2d(&tmR, obuf, nt * BN + c, row0);
+            bulk_commit_group();
+          }
+        }
+      } else if constexpr (E == Epi::Bias || E == Epi::BiasGelu) {
         if (!__all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault))) break;
         tc_fence_after();
         const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
@@ -387,8 +443,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       tc_fence_before();
       mbar_arrive(&sm->tempty[acc]);
     }
-    if constexpr (C::kTmaRes) {
-      if (lane == 0) bulk_wait_all();     // residual stores complete before the CTA exits
+    if constexpr (C::kTmaRes || C::kTmaOut) {
+      if (lane == 0) bulk_wait_all();     // the TMA stores complete before the CTA exits
     }
   }
   tc_fence_before();
@@ -461,6 +517,9 @@ cudaError_t launch_bn(const void* A, const void* W, int M, int N, int K, const E
     // the update is in place: the residual read and the output are one tensor
     if (ea.res != ea.out) return cudaErrorInvalidValue;
     e = make_map_f32_32x32(&tr, ea.out, uint64_t(M), uint64_t(N));
+    if (e != cudaSuccess) return e;
+  } else if constexpr (C::kTmaOut) {
+    e = make_map_2d(&tr, ea.out, uint64_t(M), uint64_t(N), 32);   // box 32 rows x 64 columns
     if (e != cudaSuccess) return e;
   } else {
     tr = tb;    // unused
