@@ -30,8 +30,12 @@ constexpr int BM = 128, BK = 64;
 constexpr int kThreads = 320;
 constexpr int kEpiThreads = 256;
 
-template <int BN, Epi E>
+template <int BN, Epi E, bool kPair = false>
 struct GemmCfg {
+  // kPair: two CTAs of a cluster share a 256-row tile (tcgen05.mma.cta_group::2);
+  // each loads its own 128 rows of A and half of the tile's B rows
+  static constexpr int kRowsTile = kPair ? 2 * BM : BM;
+  static constexpr int kBRows = kPair ? BN / 2 : BN;
   // the residual epilogue keeps two 32 x 32 fp32 residual tiles per epilogue
   // warp in shared memory (64 KB), paid for with a shorter operand ring
   static constexpr bool kTmaRes = E == Epi::BiasResidual && BN == 128;
@@ -39,9 +43,9 @@ struct GemmCfg {
   // from a 128-byte-swizzled 32 x 64 tile per epilogue warp (4 KB)
   static constexpr bool kTmaOut = (E == Epi::Bias || E == Epi::BiasGelu) && BN >= 128;
   static constexpr int kOutTileBytes = 32 * 128;
-  static constexpr int kStages = kTmaRes ? 4 : (BN == 256 ? 4 : 6);
+  static constexpr int kStages = kPair ? 6 : (kTmaRes ? 4 : (BN == 256 ? 4 : 6));
   static constexpr int kABytes = BM * BK * 2;        // 16 KB
-  static constexpr int kBBytes = BN * BK * 2;
+  static constexpr int kBBytes = kBRows * BK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kTmemCols = 2 * BN;           // two accumulators
   // per epilogue warp: a 32 x 32 fp32 chunk, pitch 33 (conflict-free both ways)
@@ -62,6 +66,7 @@ struct Smem {
   int abort;
 };
 static_assert(sizeof(Smem) <= 512, "the barrier block must fit its reserve in GemmCfg::kSmem");
+static_assert(GemmCfg<256, Epi::BiasResidual, true>::kSmem <= 232448, "pair config exceeds shared memory");
 
 // GELU(z) = z * Phi(z) with Phi from the erfc approximation of Abramowitz &
 // Stegun, Handbook of Mathematical Functions, formula 7.1.26 (absolute error
@@ -208,11 +213,11 @@ __device__ __forceinline__ void epilogue32_rows(const EpiArgs& ea, int row0, int
   __syncwarp();
 }
 
-template <int BN, Epi E>
+template <int BN, Epi E, bool kPair>
 __global__ void __launch_bounds__(kThreads, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                const __grid_constant__ CUtensorMap tmR, int M, int N, int K, EpiArgs ea) {
-  using C = GemmCfg<BN, E>;
+  using C = GemmCfg<BN, E, kPair>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -223,14 +228,23 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                                      C::kStagingBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m_tiles = (M + BM - 1) / BM;
+  const int m_tiles = (M + C::kRowsTile - 1) / C::kRowsTile;
   const int n_tiles = N / BN;
   const int tiles = m_tiles * n_tiles;
   const int kblocks = K / BK;
+  // a pair works through the tiles as one unit; rank 1 holds rows 128..255
+  const uint32_t rank = kPair ? cluster_ctarank() : 0u;
+  const int unit = kPair ? int(blockIdx.x >> 1) : int(blockIdx.x);
+  const int units = kPair ? int(gridDim.x >> 1) : int(gridDim.x);
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < C::kStages; ++s) { mbar_init(&sm->full[s], 1); mbar_init(&sm->empty[s], 1); }
-    for (int a = 0; a < 2; ++a) { mbar_init(&sm->tfull[a], 1); mbar_init(&sm->tempty[a], kEpiThreads); }
+    // a pair's stage is full once both producers announced their bytes and they
+    // landed; its accumulator is free once both epilogues have read it
+    for (int s = 0; s < C::kStages; ++s) { mbar_init(&sm->full[s], kPair ? 2 : 1); mbar_init(&sm->empty[s], 1); }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&sm->tfull[a], 1);
+      mbar_init(&sm->tempty[a], kPair ? 2 * (kEpiThreads / 32) : kEpiThreads);   // a pair: one per warp
+    }
     mbar_init(&sm->drain, 1);
     for (int w = 0; w < kEpiThreads / 32; ++w) { mbar_init(&sm->res_full[w][0], 1); mbar_init(&sm->res_full[w][1], 1); }
     sm->abort = 0;
@@ -241,12 +255,22 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     prefetch_tmap(&tmB);
     if constexpr (C::kTmaRes || C::kTmaOut) prefetch_tmap(&tmR);
   }
-  if (warp == 1) tmem_alloc(&sm->tmem_base, C::kTmemCols);
+  if (warp == 1) {
+    if constexpr (kPair) tmem_alloc_pair(&sm->tmem_base, C::kTmemCols);
+    else tmem_alloc(&sm->tmem_base, C::kTmemCols);
+  }
   tc_fence_before();
-  __syncthreads();
+  if constexpr (kPair) cluster_sync();   // both CTAs' barriers exist before any remote arrival
+  else __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm->tmem_base;
   volatile int* abort = &sm->abort;
+  // an abort in one CTA of a pair stops the other's waits too
+  auto abort_peer = [&]() {
+    if constexpr (kPair) {
+      if (*abort) st_cluster_u32(mapa_shared(&sm->abort, rank ^ 1u), 1u);
+    }
+  };
 
   if (warp == 0) {
     // ---------------------------------------------------------- TMA producer
@@ -254,54 +278,79 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued = 0, issued_phase = 0;    // per stage: loads in flight, their parity
-      for (int t = blockIdx.x; t < tiles && !*abort; t += gridDim.x) {
+      // a pair's loads complete on the even CTA's full barrier
+      const uint32_t full0 = kPair ? mapa_shared(&sm->full[0], 0) : 0u;
+      for (int t = unit; t < tiles && !*abort; t += units) {
         const int nt = t % n_tiles, mt = t / n_tiles;
+        const int arow = mt * C::kRowsTile + int(rank) * BM;
+        const int brow = nt * BN + int(rank) * C::kBRows;
         for (int kb = 0; kb < kblocks; ++kb) {
-          if (!mbar_wait(&sm->empty[stage], phase ^ 1, abort, ea.fault)) break;
-          mbar_arrive_expect_tx(&sm->full[stage], C::kStageBytes);
-          tma_load_2d(&tmA, sA + size_t(stage) * C::kABytes, &sm->full[stage], kb * BK, mt * BM);
-          tma_load_2d(&tmB, sB + size_t(stage) * C::kBBytes, &sm->full[stage], kb * BK, nt * BN);
+          if (!mbar_wait<kPair>(&sm->empty[stage], phase ^ 1, abort, ea.fault)) break;
+          if constexpr (kPair) {
+            const uint32_t fb = full0 + uint32_t(stage) * 8u;
+            mbar_arrive_expect_tx_relaxed_cluster(fb, C::kStageBytes);
+            tma_load_2d_pair(&tmA, sA + size_t(stage) * C::kABytes, fb, kb * BK, arow);
+            tma_load_2d_pair(&tmB, sB + size_t(stage) * C::kBBytes, fb, kb * BK, brow);
+          } else {
+            mbar_arrive_expect_tx(&sm->full[stage], C::kStageBytes);
+            tma_load_2d(&tmA, sA + size_t(stage) * C::kABytes, &sm->full[stage], kb * BK, arow);
+            tma_load_2d(&tmB, sB + size_t(stage) * C::kBBytes, &sm->full[stage], kb * BK, brow);
+          }
           issued |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
           if (++stage == C::kStages) { stage = 0; phase ^= 1; }
         }
       }
+      abort_peer();
       // every load this thread issued lands before the CTA may exit (immediate
-      // unless an aborted pipeline left loads unconsumed)
+      // unless an aborted pipeline left loads unconsumed); a pair's loads are
+      // counted on the even CTA's barriers, which its MMA thread drains
       int no_abort = 0;
-      for (int st = 0; st < C::kStages; ++st)
-        if (issued & (1u << st)) mbar_wait(&sm->full[st], (issued_phase >> st) & 1u, &no_abort, ea.fault);
+      if constexpr (!kPair) {
+        for (int st = 0; st < C::kStages; ++st)
+          if (issued & (1u << st)) mbar_wait(&sm->full[st], (issued_phase >> st) & 1u, &no_abort, ea.fault);
+      }
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------- MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16(BM, BN);
+    // (of a pair, only the even CTA issues; its commits arrive in both CTAs)
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_bf16(C::kRowsTile, BN);
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
-      for (int t = blockIdx.x; t < tiles && !*abort; t += gridDim.x, ++it) {
+      for (int t = unit; t < tiles && !*abort; t += units, ++it) {
         const int acc = it & 1;
         const uint32_t aphase = (it >> 1) & 1;
-        if (!mbar_wait(&sm->tempty[acc], aphase ^ 1, abort, ea.fault)) break;
+        if (!mbar_wait<kPair>(&sm->tempty[acc], aphase ^ 1, abort, ea.fault)) break;
         tc_fence_after();
         const uint32_t d = tmem + uint32_t(acc * BN);
         for (int kb = 0; kb < kblocks; ++kb) {
-          if (!mbar_wait(&sm->full[stage], phase, abort, ea.fault)) break;
+          if (!mbar_wait<kPair>(&sm->full[stage], phase, abort, ea.fault)) break;
           tc_fence_after();
           const uint32_t a0 = smem_u32(sA + size_t(stage) * C::kABytes);
           const uint32_t b0 = smem_u32(sB + size_t(stage) * C::kBBytes);
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)
-            mma_bf16(d, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc,
-                     (kb | k) != 0 ? 1u : 0u);
-          mma_commit(&sm->empty[stage]);
+          for (int k = 0; k < BK / 16; ++k) {
+            if constexpr (kPair)
+              mma_bf16_pair(d, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc,
+                            (kb | k) != 0 ? 1u : 0u);
+            else
+              mma_bf16(d, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc,
+                       (kb | k) != 0 ? 1u : 0u);
+          }
+          if constexpr (kPair) mma_commit_pair_both(&sm->empty[stage]);
+          else mma_commit(&sm->empty[stage]);
           if (++stage == C::kStages) { stage = 0; phase ^= 1; }
         }
-        mma_commit(&sm->tfull[acc]);
+        if constexpr (kPair) mma_commit_pair_both(&sm->tfull[acc]);
+        else mma_commit(&sm->tfull[acc]);
       }
+      abort_peer();
       // every MMA issued has completed before the tensor memory is released
       int no_abort = 0;
-      mma_commit(&sm->drain);
+      if constexpr (kPair) mma_commit_pair_local(&sm->drain);
+      else mma_commit(&sm->drain);
       mbar_wait(&sm->drain, 0, &no_abort, ea.fault);
     }
   } else {
@@ -310,14 +359,15 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const int half = (warp - 2) >> 2;       // which half of the tile's columns
     constexpr int kW = BN / 2 >= 64 ? 64 : 32;    // bf16 epilogue step (columns)
     int it = 0;
-    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++it) {
+    const uint32_t tempty0 = kPair ? mapa_shared(&sm->tempty[0], 0) : 0u;
+    for (int t = unit; t < tiles; t += units, ++it) {
       const int nt = t % n_tiles, mt = t / n_tiles;
       const int acc = it & 1;
       const uint32_t aphase = (it >> 1) & 1;
-      const int row0 = mt * BM + q * 32;
+      const int row0 = mt * C::kRowsTile + int(rank) * BM + q * 32;
       const int c_begin = half * (BN / 2), c_end = (half + 1) * (BN / 2);
       if constexpr (C::kTmaOut) {
-        if (!__all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault))) break;
+        if (!__all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault))) break;
         tc_fence_after();
         const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
         unsigned char* obuf = reinterpret_cast<unsigned char*>(staging) +
@@ -347,7 +397,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           }
         }
       } else if constexpr (E == Epi::Bias || E == Epi::BiasGelu) {
-        if (!__all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault))) break;
+        if (!__all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault))) break;
         tc_fence_after();
         const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
 #pragma unroll 1
@@ -377,7 +427,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           }
         }
         const uint32_t rph = uint32_t(it) & 1u;
-        bool ok = __all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault));
+        bool ok = __all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault));
         if (ok) {
           tc_fence_after();
           const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
@@ -427,7 +477,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         // the first chunk's residual loads overlap the wait for the accumulator
         float rv[32];
         load_residual(ea, row0, M, nt * BN + c_begin, N, lane, rv);
-        if (!__all_sync(0xffffffffu, mbar_wait(&sm->tfull[acc], aphase, abort, ea.fault))) break;
+        if (!__all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault))) break;
         tc_fence_after();
         const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
 #pragma unroll 1
@@ -441,17 +491,28 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         }
       }
       tc_fence_before();
-      mbar_arrive(&sm->tempty[acc]);
+      if constexpr (kPair) {
+        __syncwarp();
+        if (lane == 0) {
+          if (rank == 0) mbar_arrive(&sm->tempty[acc]);
+          else mbar_arrive_cluster(tempty0 + uint32_t(acc) * 8u);
+        }
+      } else {
+        mbar_arrive(&sm->tempty[acc]);
+      }
     }
+    if (lane == 0) abort_peer();
     if constexpr (C::kTmaRes || C::kTmaOut) {
       if (lane == 0) bulk_wait_all();     // the TMA stores complete before the CTA exits
     }
   }
   tc_fence_before();
-  __syncthreads();
+  if constexpr (kPair) cluster_sync();   // neither CTA leaves while the other may still signal it
+  else __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, C::kTmemCols);
+    if constexpr (kPair) tmem_dealloc_pair(tmem, C::kTmemCols);
+    else tmem_dealloc(tmem, C::kTmemCols);
   }
 }
 
@@ -504,14 +565,14 @@ cudaError_t make_map_f32_32x32(CUtensorMap* map, const void* ptr, uint64_t rows,
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <int BN, Epi E>
+template <int BN, Epi E, bool kPair>
 cudaError_t launch_bn(const void* A, const void* W, int M, int N, int K, const EpiArgs& ea,
                       cudaStream_t s) {
-  using C = GemmCfg<BN, E>;
+  using C = GemmCfg<BN, E, kPair>;
   CUtensorMap ta, tb, tr;
   cudaError_t e = make_map_2d(&ta, A, uint64_t(M), uint64_t(K), BM);
   if (e != cudaSuccess) return e;
-  e = make_map_2d(&tb, W, uint64_t(N), uint64_t(K), BN);
+  e = make_map_2d(&tb, W, uint64_t(N), uint64_t(K), C::kBRows);
   if (e != cudaSuccess) return e;
   if constexpr (C::kTmaRes) {
     // the update is in place: the residual read and the output are one tensor
@@ -524,34 +585,66 @@ cudaError_t launch_bn(const void* A, const void* W, int M, int N, int K, const E
   } else {
     tr = tb;    // unused
   }
-  static bool attr_set = false;
-  if (!attr_set) {
-    e = cudaFuncSetAttribute(gemm_tc_kernel<BN, E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             int(C::kSmem));
+  auto kernel = gemm_tc_kernel<BN, E, kPair>;
+  static int max_units = 0;     // CTAs (or CTA pairs) resident at once
+  if (max_units == 0) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(C::kSmem));
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    if (g_num_sms == 0) {
+      int dev = 0;
+      cudaGetDevice(&dev);
+      cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+    }
+    if constexpr (kPair) {
+      cudaLaunchConfig_t cfg = {};
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = 2; at[0].val.clusterDim.y = 1; at[0].val.clusterDim.z = 1;
+      cfg.gridDim = dim3(unsigned(g_num_sms & ~1));
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = C::kSmem;
+      cfg.attrs = at;
+      cfg.numAttrs = 1;
+      int clusters = 0;
+      e = cudaOccupancyMaxActiveClusters(&clusters, kernel, &cfg);
+      if (e != cudaSuccess) return e;
+      if (clusters < 1) return cudaErrorInvalidConfiguration;
+      max_units = clusters;
+    } else {
+      max_units = g_num_sms;
+    }
   }
-  if (g_num_sms == 0) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+  const int tiles = ((M + C::kRowsTile - 1) / C::kRowsTile) * (N / BN);
+  const int units = tiles < max_units ? tiles : max_units;
+  if constexpr (kPair) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2; at[0].val.clusterDim.y = 1; at[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(unsigned(2 * units));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = C::kSmem;
+    cfg.stream = s;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, ta, tb, tr, M, N, K, ea);
+  } else {
+    kernel<<<units, kThreads, C::kSmem, s>>>(ta, tb, tr, M, N, K, ea);
+    return cudaGetLastError();
   }
-  const int tiles = ((M + BM - 1) / BM) * (N / BN);
-  const int grid = tiles < g_num_sms ? tiles : g_num_sms;
-  gemm_tc_kernel<BN, E><<<grid, kThreads, C::kSmem, s>>>(ta, tb, tr, M, N, K, ea);
-  return cudaGetLastError();
 }
 
-template <int BN>
+template <int BN, bool kPair>
 cudaError_t launch_epi(Epi epi, const void* A, const void* W, int M, int N, int K,
                        const EpiArgs& ea, cudaStream_t s) {
   switch (epi) {
-    case Epi::Bias: return launch_bn<BN, Epi::Bias>(A, W, M, N, K, ea, s);
-    case Epi::BiasGelu: return launch_bn<BN, Epi::BiasGelu>(A, W, M, N, K, ea, s);
-    case Epi::BiasResidualScatter: return launch_bn<BN, Epi::BiasResidualScatter>(A, W, M, N, K, ea, s);
+    case Epi::Bias: return launch_bn<BN, Epi::Bias, kPair>(A, W, M, N, K, ea, s);
+    case Epi::BiasGelu: return launch_bn<BN, Epi::BiasGelu, kPair>(A, W, M, N, K, ea, s);
+    case Epi::BiasResidualScatter:
+      return launch_bn<BN, Epi::BiasResidualScatter, kPair>(A, W, M, N, K, ea, s);
     case Epi::BiasResidual:
       // BN = 128 is the TMA residual epilogue, chosen in launch_gemm_tc
-      if constexpr (BN != 128) return launch_bn<BN, Epi::BiasResidual>(A, W, M, N, K, ea, s);
+      if constexpr (BN != 128) return launch_bn<BN, Epi::BiasResidual, kPair>(A, W, M, N, K, ea, s);
       break;
   }
   return cudaErrorInvalidValue;
@@ -562,18 +655,19 @@ cudaError_t launch_epi(Epi epi, const void* A, const void* W, int M, int N, int 
 cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* W, int M, int N, int K,
                            const EpiArgs& ea, cudaStream_t s) {
   if (M < 1 || K % BK != 0 || N % 64 != 0) return cudaErrorInvalidValue;
+  // tiles 128 or 256 columns wide run on CTA pairs (256-row tiles); 64-wide on single CTAs
   if (epi == Epi::BiasResidual) {
     // a short mainloop (K <= 2048) cannot hide the fp32 residual traffic behind
     // the MMAs: 128-column tiles with the TMA residual epilogue; a long one keeps
     // 256-column tiles and the register epilogue
     if (N % 128 == 0 && (K <= 2048 || N % 256 != 0))
-      return launch_bn<128, Epi::BiasResidual>(A, W, M, N, K, ea, s);
-    if (N % 256 == 0) return launch_epi<256>(epi, A, W, M, N, K, ea, s);
-    return launch_epi<64>(epi, A, W, M, N, K, ea, s);
+      return launch_bn<128, Epi::BiasResidual, true>(A, W, M, N, K, ea, s);
+    if (N % 256 == 0) return launch_epi<256, true>(epi, A, W, M, N, K, ea, s);
+    return launch_epi<64, false>(epi, A, W, M, N, K, ea, s);
   }
-  if (N % 256 == 0) return launch_epi<256>(epi, A, W, M, N, K, ea, s);
-  if (N % 128 == 0) return launch_epi<128>(epi, A, W, M, N, K, ea, s);
-  return launch_epi<64>(epi, A, W, M, N, K, ea, s);
+  if (N % 256 == 0) return launch_epi<256, true>(epi, A, W, M, N, K, ea, s);
+  if (N % 128 == 0) return launch_epi<128, true>(epi, A, W, M, N, K, ea, s);
+  return launch_epi<64, false>(epi, A, W, M, N, K, ea, s);
 }
 
 }  // namespace sr
