@@ -49,6 +49,13 @@ size_t align_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
 void sr::set_error_message(const std::string& msg) { g_last_msg = msg; }
 
 namespace {
+thread_local bool g_pdl = false;
+}  // namespace
+bool sr::pdl_enabled() { return g_pdl; }
+sr::PdlScope::PdlScope(bool on) : prev(g_pdl) { g_pdl = on; }
+sr::PdlScope::~PdlScope() { g_pdl = prev; }
+
+namespace {
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
@@ -378,6 +385,9 @@ sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, flo
     SR_CUDA(sr::launch_widen(h->dt, x, xs, n, s), "widen x");
   }
   sr_status st;
+  // every later kernel of the forward may start while its predecessor finishes
+  // (not while tracing, which records events between kernels)
+  const sr::PdlScope pdl(!h->trace);
   // stage 1: dense early
   for (int i = 0; i < c.n1; ++i)
     if ((st = run_block(h, xs, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;

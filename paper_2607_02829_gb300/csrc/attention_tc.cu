@@ -115,6 +115,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
   tc_fence_after();
   const uint32_t tmem = sm->tmem_base;
   volatile int* abort = &sm->abort;
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
 
   if (warp < 4) {
     // registers: 56 per thread for the load / MMA warpgroup, 224 for the two
@@ -403,9 +405,8 @@ cudaError_t launch_attention_tc(const void* qkv, void* out, int B, int T, int he
     attr_set = true;
   }
   const int grid = B * heads * ((T + kBQ - 1) / kBQ);
-  attention_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(tm, static_cast<bf16*>(out), T, heads,
-                                                         fault);
-  return cudaGetLastError();
+  return launch_k(attention_tc_kernel, dim3(grid), dim3(kThreads), kSmemBytes, s, 1, tm,
+                  static_cast<bf16*>(out), T, heads, fault);
 }
 
 }  // namespace sr

@@ -9,6 +9,14 @@ namespace sr {
 
 using bf16 = __nv_bfloat16;
 
+// Programmatic dependent launch, device side: wait until the grids this one
+// depends on have completed and their writes are visible (a no-op for a
+// kernel launched without the attribute); then let the next grid launch.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // Element-type traits: the library computes in fp32 and stores fp32 or bf16.
 template <typename T> struct Elem;
 template <> struct Elem<float> {

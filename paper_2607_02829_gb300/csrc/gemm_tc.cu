@@ -265,6 +265,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   tc_fence_after();
   const uint32_t tmem = sm->tmem_base;
   volatile int* abort = &sm->abort;
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
   // an abort in one CTA of a pair stops the other's waits too
   auto abort_peer = [&]() {
     if constexpr (kPair) {
@@ -616,22 +618,8 @@ cudaError_t launch_bn(const void* A, const void* W, int M, int N, int K, const E
   }
   const int tiles = ((M + C::kRowsTile - 1) / C::kRowsTile) * (N / BN);
   const int units = tiles < max_units ? tiles : max_units;
-  if constexpr (kPair) {
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute at[1];
-    at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = 2; at[0].val.clusterDim.y = 1; at[0].val.clusterDim.z = 1;
-    cfg.gridDim = dim3(unsigned(2 * units));
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = C::kSmem;
-    cfg.stream = s;
-    cfg.attrs = at;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kernel, ta, tb, tr, M, N, K, ea);
-  } else {
-    kernel<<<units, kThreads, C::kSmem, s>>>(ta, tb, tr, M, N, K, ea);
-    return cudaGetLastError();
-  }
+  return launch_k(kernel, dim3(unsigned(kPair ? 2 * units : units)), dim3(kThreads), C::kSmem, s,
+                  kPair ? 2u : 1u, ta, tb, tr, M, N, K, ea);
 }
 
 template <int BN, bool kPair>

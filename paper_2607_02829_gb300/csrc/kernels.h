@@ -10,6 +10,47 @@ namespace sr {
 
 enum class DType : int { F32 = 0, BF16 = 1 };
 
+// ---- programmatic dependent launch -----------------------------------------
+// While a PdlScope is alive on the calling thread, the launchers below mark
+// each kernel as allowed to start while the previous kernel of the stream is
+// still finishing.  Such a kernel runs its setup (barriers, tensor memory,
+// tensor-map prefetch) early, and every thread waits (griddepcontrol.wait)
+// for the previous grids to complete before it touches global memory.
+bool pdl_enabled();
+struct PdlScope {
+  explicit PdlScope(bool on);
+  ~PdlScope();
+  PdlScope(const PdlScope&) = delete;
+  PdlScope& operator=(const PdlScope&) = delete;
+  bool prev;
+};
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                            cudaStream_t s, unsigned cluster, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute at[2];
+  unsigned n = 0;
+  if (pdl_enabled()) {
+    at[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  if (cluster > 1) {
+    at[n].id = cudaLaunchAttributeClusterDimension;
+    at[n].val.clusterDim.x = cluster;
+    at[n].val.clusterDim.y = 1;
+    at[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = at;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 // ---- token selection (Sec. 3.2; App. B.2) --------------------------------
 // Random: K smallest SplitMix64 keys per sample (ties by index), sorted indices.
 cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared,

@@ -14,6 +14,8 @@ template <int NV>
 __global__ void __launch_bounds__(256)
 gather_rows_kernel(const float* __restrict__ x, const int32_t* __restrict__ idx, int L, int K,
                    int D, int rows, float* __restrict__ h) {
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
   constexpr int V = 4;
   const int lane = threadIdx.x & 31;
   const int nv = D / V;
@@ -41,6 +43,8 @@ template <typename T, int NV>
 __global__ void __launch_bounds__(256)
 layernorm_kernel(const float* __restrict__ x, const T* __restrict__ g, const T* __restrict__ bta,
                  T* __restrict__ y, int rows, int D, float eps) {
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
   constexpr int V = Elem<T>::kVec;
   const int lane = threadIdx.x & 31;
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -95,14 +99,15 @@ cudaError_t gather_t(const float* x, const int32_t* idx, int B, int L, int K, in
   const int rows = B * K;
   int blocks = (rows + 7) / 8;
   if (blocks > 152 * 16) blocks = 152 * 16;
-  gather_rows_kernel<NV><<<blocks, 256, 0, s>>>(x, idx, L, K, D, rows, h);
-  return cudaGetLastError();
+  return launch_k(gather_rows_kernel<NV>, dim3(blocks), dim3(256), 0, s, 1, x, idx, L, K, D, rows, h);
 }
 
 // Storage dtype <-> fp32 stream, n elements (n % 8 == 0), 16-byte vectors.
 template <typename T>
 __global__ void __launch_bounds__(256)
 widen_kernel(const T* __restrict__ x, float* __restrict__ y, size_t nvec) {
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
   constexpr int V = Elem<T>::kVec;
   for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
        i += size_t(gridDim.x) * blockDim.x) {
@@ -117,6 +122,8 @@ widen_kernel(const T* __restrict__ x, float* __restrict__ y, size_t nvec) {
 template <typename T>
 __global__ void __launch_bounds__(256)
 narrow_kernel(const float* __restrict__ x, T* __restrict__ y, size_t nvec) {
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
   constexpr int V = Elem<T>::kVec;
   for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
        i += size_t(gridDim.x) * blockDim.x) {
@@ -139,10 +146,9 @@ int grid_for(size_t nvec) {
 template <typename T, int NV>
 cudaError_t layernorm_t(const float* x, const void* g, const void* b, void* y, int rows, int D,
                         float eps, cudaStream_t s) {
-  layernorm_kernel<T, NV><<<(rows + 7) / 8, 256, 0, s>>>(
-      x, static_cast<const T*>(g), static_cast<const T*>(b),
-      static_cast<T*>(y), rows, D, eps);
-  return cudaGetLastError();
+  return launch_k(layernorm_kernel<T, NV>, dim3((rows + 7) / 8), dim3(256), 0, s, 1, x,
+                  static_cast<const T*>(g), static_cast<const T*>(b), static_cast<T*>(y), rows, D,
+                  eps);
 }
 
 // vectors per lane needed for a row of D elements
@@ -164,23 +170,23 @@ cudaError_t launch_gather_rows(const float* x, const int32_t* idx, int B, int L,
 cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream_t s) {
   if (dt == DType::BF16) {
     const size_t nvec = n / 8;
-    widen_kernel<bf16><<<grid_for(nvec), 256, 0, s>>>(static_cast<const bf16*>(x), y, nvec);
-  } else {
-    const size_t nvec = n / 4;
-    widen_kernel<float><<<grid_for(nvec), 256, 0, s>>>(static_cast<const float*>(x), y, nvec);
+    return launch_k(widen_kernel<bf16>, dim3(grid_for(nvec)), dim3(256), 0, s, 1,
+                    static_cast<const bf16*>(x), y, nvec);
   }
-  return cudaGetLastError();
+  const size_t nvec = n / 4;
+  return launch_k(widen_kernel<float>, dim3(grid_for(nvec)), dim3(256), 0, s, 1,
+                  static_cast<const float*>(x), y, nvec);
 }
 
 cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStream_t s) {
   if (dt == DType::BF16) {
     const size_t nvec = n / 8;
-    narrow_kernel<bf16><<<grid_for(nvec), 256, 0, s>>>(x, static_cast<bf16*>(y), nvec);
-  } else {
-    const size_t nvec = n / 4;
-    narrow_kernel<float><<<grid_for(nvec), 256, 0, s>>>(x, static_cast<float*>(y), nvec);
+    return launch_k(narrow_kernel<bf16>, dim3(grid_for(nvec)), dim3(256), 0, s, 1, x,
+                    static_cast<bf16*>(y), nvec);
   }
-  return cudaGetLastError();
+  const size_t nvec = n / 4;
+  return launch_k(narrow_kernel<float>, dim3(grid_for(nvec)), dim3(256), 0, s, 1, x,
+                  static_cast<float*>(y), nvec);
 }
 
 cudaError_t launch_layernorm(DType dt, const float* x, const void* g, const void* b, void* y,

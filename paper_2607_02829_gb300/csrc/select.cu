@@ -132,6 +132,9 @@ __device__ void select_smallest_sorted(const Key* keys, int L, int K, int32_t* o
 __global__ void __launch_bounds__(kSelThreads)
 select_random_kernel(int L, int K, uint64_t seed, int shared, int32_t* idx) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
+
   uint64_t* keys = reinterpret_cast<uint64_t*>(smem_raw);
   const int b = blockIdx.x;
   const uint64_t bb = shared ? 0ull : uint64_t(b);
@@ -146,6 +149,9 @@ select_random_kernel(int L, int K, uint64_t seed, int shared, int32_t* idx) {
 __global__ void __launch_bounds__(kSelThreads)
 select_topk_kernel(int L, int K, const float* __restrict__ score, int32_t* idx) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
+
   uint32_t* keys = reinterpret_cast<uint32_t*>(smem_raw);
   const int b = blockIdx.x;
   for (int i = threadIdx.x; i < L; i += blockDim.x) keys[i] = desc_key(score[size_t(b) * L + i]);
@@ -158,6 +164,8 @@ select_topk_kernel(int L, int K, const float* __restrict__ score, int32_t* idx) 
 template <typename T>
 __global__ void __launch_bounds__(256)
 token_sq_norms_kernel(const float* __restrict__ x, int rows, int D, float* __restrict__ score) {
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= rows) return;
@@ -187,8 +195,8 @@ cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared,
   cudaError_t e = cudaFuncSetAttribute(select_random_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
-  select_random_kernel<<<B, kSelThreads, smem, s>>>(L, K, seed, shared, idx);
-  return cudaGetLastError();
+  return launch_k(select_random_kernel, dim3(B), dim3(kSelThreads), smem, s, 1, L, K, seed, shared,
+                  idx);
 }
 
 cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t* idx,
@@ -197,18 +205,15 @@ cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t*
   cudaError_t e = cudaFuncSetAttribute(select_topk_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
-  select_topk_kernel<<<B, kSelThreads, smem, s>>>(L, K, score, idx);
-  return cudaGetLastError();
+  return launch_k(select_topk_kernel, dim3(B), dim3(kSelThreads), smem, s, 1, L, K, score, idx);
 }
 
 cudaError_t launch_token_sq_norms(DType dt, const float* x, int rows, int D, float* score,
                                   cudaStream_t s) {
   const int blocks = (rows + 7) / 8;
   if (dt == DType::BF16)
-    token_sq_norms_kernel<bf16><<<blocks, 256, 0, s>>>(x, rows, D, score);
-  else
-    token_sq_norms_kernel<float><<<blocks, 256, 0, s>>>(x, rows, D, score);
-  return cudaGetLastError();
+    return launch_k(token_sq_norms_kernel<bf16>, dim3(blocks), dim3(256), 0, s, 1, x, rows, D, score);
+  return launch_k(token_sq_norms_kernel<float>, dim3(blocks), dim3(256), 0, s, 1, x, rows, D, score);
 }
 
 }  // namespace sr
