@@ -351,7 +351,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--split", default=None,
                     help="override the block split n1,n2,n3 (kernel studies and profiling)")
-    ap.add_argument("--sweep", choices=["gather"], default=None,
+    ap.add_argument("--sweep", choices=["gather", "ensemble"], default=None,
                     help="size sweep of one kernel (prints one JSON line per size)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -364,6 +364,8 @@ def main():
         return run_reference(args, rank, world)
     if args.sweep == "gather":
         return gather_sweep(args)
+    if args.sweep == "ensemble":
+        return ensemble_sweep(args)
 
     import torch
     import torch.distributed as dist
@@ -460,6 +462,56 @@ def gather_sweep(args):
         enc.close()
         del x, out
         torch.cuda.empty_cache()
+
+
+def ensemble_sweep(args):
+    """Implicit ensembling on the workload (default 0.25 deg): M = 1, 2, 4, 8
+    members with different seeds through sr_forward_ensemble (dense-early blocks
+    once) against M separate sr_forward calls; CUDA-event time per ensemble with
+    L2 flushed before each, inputs resident in HBM."""
+    import torch
+    from paper_2607_02829_gb300 import binding as b, build
+    build.build()
+    wl = _workload(args.workload, args.split)
+    x, ws = rank_inputs(wl, 0)
+    cfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, wl.n1, wl.n2, wl.n3, dtype=wl.dtype,
+                        selector=wl.selector)
+    enc = b.Encoder(cfg, max_keep_ratio=wl.keep_ratio)
+    xd = x.cuda()
+    warr = b.weights_array([{k: v.cuda() for k, v in blk.items()} for blk in ws])
+    out = torch.empty_like(xd)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    s = torch.cuda.current_stream()
+
+    def timed(fn):
+        for _ in range(args.warmup):
+            fn()
+        tot = 0.0
+        for _ in range(args.steps):
+            flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(s)
+            fn()
+            e1.record(s)
+            torch.cuda.synchronize()
+            tot += e0.elapsed_time(e1)
+        return tot / args.steps
+
+    for M in (1, 2, 4, 8):
+        seeds = [wl.select_seed + 17 * m for m in range(M)]
+        ens_ms = timed(lambda: enc.forward_ensemble(xd, warr, wl.keep_ratio, seeds, out=out))
+
+        def separate():
+            for sd in seeds:
+                b.sr_forward(enc.handle, xd.data_ptr(), warr, wl.keep_ratio, sd, out.data_ptr(),
+                             None, s.cuda_stream)
+        sep_ms = timed(separate)
+        print(json.dumps({"sweep": "ensemble", "workload": wl.name, "members": M,
+                          "ms_per_ensemble": ens_ms, "ms_separate_forwards": sep_ms,
+                          "speedup_vs_separate": sep_ms / ens_ms,
+                          "member_tokens_per_s": wl.B * wl.L * M / (ens_ms * 1e-3)}), flush=True)
+    enc.close()
 
 
 def run_reference(args, rank, world):

@@ -127,6 +127,27 @@ sr_status sr_select(sr_handle* h, const void* x, float keep_ratio, uint64_t seed
 sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, float keep_ratio,
                      uint64_t seed, void* out, int32_t* idx_out, void* stream);
 
+/* Implicit ensemble (Sec. 3, "Training and inference"; App. B): averaging the
+ * outputs of forward passes with different selection seeds.  Member m is
+ * exactly sr_forward(x, seeds[m]); the n1 dense-early blocks do not depend on
+ * the seed, so they run once and their result is reused by every member.
+ *  seeds        : HOST array of M >= 1 selection seeds.
+ *  ens_workspace: device buffer of at least sr_ensemble_workspace_bytes(cfg)
+ *                 bytes, 256-byte aligned, caller-owned (the dense-early result
+ *                 and the fp32 sum of the members).
+ *  out          : [B, L, D] device; the mean over the members of their fp32
+ *                 results, rounded once to the storage dtype.  May equal x.
+ *  members_out  : optional [M, B, L, D] device; member m's output, bit-identical
+ *                 to sr_forward's for seed seeds[m].  NULL to skip.
+ *  idx_out      : optional [M, B, K] int32 device; member m's index set.
+ * Errors as sr_forward, plus SR_ERR_INVALID_ARG for M < 1 or NULL seeds and
+ * SR_ERR_WORKSPACE for a missing or short ensemble workspace. */
+size_t sr_ensemble_workspace_bytes(const sr_config* cfg);
+sr_status sr_forward_ensemble(sr_handle* h, const void* x, const sr_block_weights* w,
+                              float keep_ratio, const uint64_t* seeds, int32_t M,
+                              void* ens_workspace, size_t ens_ws_bytes, void* out,
+                              void* members_out, int32_t* idx_out, void* stream);
+
 /* sr_forward from and to HOST memory: copies x_host ([B, L, D], preferably
  * pinned) into the caller's device buffer `dev_xout`, runs sr_forward in place
  * on it, and copies the result back into out_host.  All three steps are

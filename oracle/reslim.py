@@ -248,6 +248,23 @@ def forward(x: np.ndarray, weights: Sequence[Dict[str, np.ndarray]], n1: int, n2
     return x, idx
 
 
+def forward_ensemble(x: np.ndarray, weights: Sequence[Dict[str, np.ndarray]], n1: int, n2: int,
+                     n3: int, heads: int, keep_ratio: float, seeds: Sequence[int],
+                     selector: str = "random", shared_indices: bool = False, eps: float = 1e-5,
+                     threads: int = 0):
+    """Implicit ensembling (Sec. 3, "Training and inference"; App. B): the mean
+    of the routed forward over a set of selection seeds, each member a plain
+    call of ``forward``.  Returns (mean, [member outputs], [member index sets]).
+    """
+    outs, idxs = [], []
+    for seed in seeds:
+        y, idx = forward(x, weights, n1, n2, n3, heads, keep_ratio, seed=seed, selector=selector,
+                         shared_indices=shared_indices, eps=eps, threads=threads)
+        outs.append(y)
+        idxs.append(idx)
+    return sum(outs) / float(len(outs)), outs, idxs
+
+
 def dense_stack(x: np.ndarray, weights: Sequence[Dict[str, np.ndarray]], heads: int,
                 eps: float = 1e-5, threads: int = 0) -> np.ndarray:
     """All blocks on all tokens: the dense baseline (routing disabled)."""

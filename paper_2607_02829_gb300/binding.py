@@ -75,6 +75,12 @@ def lib() -> ctypes.CDLL:
         L.sr_forward_host.argtypes = [vp, vp, ctypes.POINTER(sr_block_weights), ctypes.c_float,
                                       ctypes.c_uint64, vp, vp, vp, vp]
         L.sr_forward_host.restype = st
+        L.sr_ensemble_workspace_bytes.argtypes = [ctypes.POINTER(sr_config)]
+        L.sr_ensemble_workspace_bytes.restype = sz
+        L.sr_forward_ensemble.argtypes = [vp, vp, ctypes.POINTER(sr_block_weights), ctypes.c_float,
+                                          ctypes.POINTER(ctypes.c_uint64), i32, vp, sz, vp, vp, vp,
+                                          vp]
+        L.sr_forward_ensemble.restype = st
         L.sr_destroy.argtypes = [vp]; L.sr_destroy.restype = st
         L.sr_trace_enable.argtypes = [vp, ctypes.c_int]; L.sr_trace_enable.restype = st
         L.sr_trace_read.argtypes = [vp, ctypes.POINTER(sr_trace_entry), ctypes.c_int]
@@ -130,6 +136,19 @@ def sr_forward_host(handle: int, x_host: int, weights: ctypes.Array, keep_ratio:
                     stream: int) -> None:
     _check(lib().sr_forward_host(handle, x_host, weights, keep_ratio, seed % (1 << 64), dev_xout,
                                  out_host, idx_out, stream), "sr_forward_host")
+
+
+def sr_ensemble_workspace_bytes(cfg: sr_config) -> int:
+    return int(lib().sr_ensemble_workspace_bytes(ctypes.byref(cfg)))
+
+
+def sr_forward_ensemble(handle: int, x: int, weights: ctypes.Array, keep_ratio: float,
+                        seeds: Sequence[int], ens_ws: int, ens_ws_bytes: int, out: int,
+                        members_out: Optional[int], idx_out: Optional[int], stream: int) -> None:
+    arr = (ctypes.c_uint64 * max(len(seeds), 1))(*[int(v) % (1 << 64) for v in seeds])
+    _check(lib().sr_forward_ensemble(handle, x, weights, keep_ratio, arr, len(seeds), ens_ws,
+                                     ens_ws_bytes, out, members_out, idx_out, stream),
+           "sr_forward_ensemble")
 
 
 def sr_destroy(handle: Optional[int]) -> None:
@@ -231,3 +250,26 @@ class Encoder:
         sr_forward(self.handle, x.data_ptr(), weights, keep_ratio, seed, out.data_ptr(),
                    idx.data_ptr() if idx is not None else None, s.cuda_stream)
         return out, idx
+
+    def forward_ensemble(self, x, weights: ctypes.Array, keep_ratio, seeds, out=None,
+                         want_members=False, want_idx=False, stream=None):
+        """Mean over len(seeds) members (see sr_forward_ensemble); returns
+        (out, members [M, B, L, D] or None, idx [M, B, K] or None)."""
+        import torch
+        M = len(seeds)
+        nbytes = sr_ensemble_workspace_bytes(self.cfg)
+        if getattr(self, "ens_ws", None) is None or self.ens_ws.numel() < nbytes + 256:
+            self.ens_ws = torch.empty(nbytes + 256, dtype=torch.uint8, device="cuda")
+        ptr = (self.ens_ws.data_ptr() + 255) // 256 * 256
+        if out is None:
+            out = torch.empty_like(x)
+        members = torch.empty((M,) + tuple(x.shape), dtype=x.dtype, device="cuda") if want_members else None
+        idx = None
+        if want_idx:
+            K = sr_keep_count(self.cfg.L, keep_ratio)
+            idx = torch.empty((M, self.cfg.B, max(K, 1)), dtype=torch.int32, device="cuda")
+        s = stream if stream is not None else torch.cuda.current_stream()
+        sr_forward_ensemble(self.handle, x.data_ptr(), weights, keep_ratio, seeds, ptr, nbytes,
+                            out.data_ptr(), members.data_ptr() if members is not None else None,
+                            idx.data_ptr() if idx is not None else None, s.cuda_stream)
+        return out, members, idx

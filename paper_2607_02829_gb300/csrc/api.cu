@@ -349,8 +349,11 @@ sr_status sr_select(sr_handle* h, const void* x, float keep_ratio, uint64_t seed
   return do_select(h, xs, K, seed, idx, s);
 }
 
-sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, float keep_ratio,
-                     uint64_t seed, void* out, int32_t* idx_out, void* stream) {
+namespace {
+
+// Host checks shared by sr_forward and sr_forward_ensemble (no CUDA calls).
+sr_status check_forward_args(const sr_handle* h, const void* x, const sr_block_weights* w,
+                             float keep_ratio, const void* out, int32_t* K) {
   if (!h) return fail(SR_ERR_INVALID_ARG, "handle is NULL");
   const sr_config& c = h->cfg;
   const int N = c.n1 + c.n2 + c.n3;
@@ -359,43 +362,57 @@ sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, flo
   if (!w) return fail(SR_ERR_INVALID_ARG, "weights array is NULL");
   for (int i = 0; i < N; ++i)
     if (!weights_ok(w[i])) return fail(SR_ERR_INVALID_ARG, "a block weight pointer is NULL or misaligned");
-  if (idx_out && !aligned(idx_out, 4)) return fail(SR_ERR_INVALID_ARG, "idx_out misaligned");
-  const int32_t K = keep_count(c.L, keep_ratio);
-  if (K < 0) return fail(SR_ERR_INVALID_ARG, "keep_ratio must lie in (0, 1]");
+  *K = keep_count(c.L, keep_ratio);
+  if (*K < 0) return fail(SR_ERR_INVALID_ARG, "keep_ratio must lie in (0, 1]");
   const bool route = keep_ratio < 1.0f && c.n2 > 0;
-  if (K < 1 && (route || idx_out)) return fail(SR_ERR_INVALID_ARG, "K = floor(L * keep_ratio) is 0");
-  if (route && K > h->Kmax) return fail(SR_ERR_WORKSPACE, "K exceeds the workspace's routed capacity");
+  if (*K < 1 && route) return fail(SR_ERR_INVALID_ARG, "K = floor(L * keep_ratio) is 0");
+  if (route && *K > h->Kmax) return fail(SR_ERR_WORKSPACE, "K exceeds the workspace's routed capacity");
   if (!route && c.n2 > 0 && size_t(c.B) * c.L > h->plan.block_rows)
     return fail(SR_ERR_WORKSPACE, "workspace sized for keep ratios below 1 only");
   const size_t bytes = size_t(c.B) * c.L * c.D * h->es;
   const char* xb = static_cast<const char*>(x);
-  char* ob = static_cast<char*>(out);
+  const char* ob = static_cast<const char*>(out);
   if (xb != ob && xb < ob + bytes && ob < xb + bytes)
     return fail(SR_ERR_INVALID_ARG, "out partially overlaps x");
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  return SR_OK;
+}
+
+// x (storage dtype) into the fp32 stream xs, then the n1 dense-early blocks.
+sr_status widen_and_early(sr_handle* h, const void* x, const sr_block_weights* w, float* xs,
+                          cudaStream_t s) {
+  const sr_config& c = h->cfg;
   if (!h->fault_cleared) {
     SR_CUDA(cudaMemsetAsync(h->fault(), 0, sizeof(unsigned int), s), "clear fault word");
     h->fault_cleared = true;
   }
   const size_t n = size_t(c.B) * c.L * c.D;
-  float* xs = static_cast<float*>(h->at(h->plan.xs));
   {
     // the residual stream is held in fp32 for the whole forward
-    TraceScope t(h, SR_KERN_COPY, 0.0, double(bytes) + 4.0 * n, s);
+    TraceScope t(h, SR_KERN_COPY, 0.0, double(n) * (h->es + 4.0), s);
     SR_CUDA(sr::launch_widen(h->dt, x, xs, n, s), "widen x");
   }
-  sr_status st;
-  // every later kernel of the forward may start while its predecessor finishes
-  // (not while tracing, which records events between kernels)
+  // every later kernel may start while its predecessor finishes (not while
+  // tracing, which records events between kernels)
   const sr::PdlScope pdl(!h->trace);
-  // stage 1: dense early
+  sr_status st;
   for (int i = 0; i < c.n1; ++i)
     if ((st = run_block(h, xs, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
+  return SR_OK;
+}
+
+// Everything after the dense-early blocks, in place on the fp32 stream xs:
+// selection, gather, the sparse middle with the delta scatter fused into its
+// last block, and the dense-late blocks (Alg. 1 after its dense-early loop).
+sr_status route_and_late(sr_handle* h, float* xs, const sr_block_weights* w, float keep_ratio,
+                         int32_t K, uint64_t seed, int32_t* idx_out, cudaStream_t s) {
+  const sr_config& c = h->cfg;
+  const int N = c.n1 + c.n2 + c.n3;
+  const bool route = keep_ratio < 1.0f && c.n2 > 0;
+  sr_status st;
   int32_t* idx = idx_out ? idx_out : static_cast<int32_t*>(h->at(h->plan.idx));
   if (route || idx_out)
     if ((st = do_select(h, xs, K, seed, idx, s)) != SR_OK) return st;
   if (route) {
-    // stage 2: gather, sparse middle, delta scatter in the last block's epilogue
     float* hs = static_cast<float*>(h->at(h->plan.hs));
     {
       TraceScope t(h, SR_KERN_GATHER, 0.0, 8.0 * c.B * K * c.D + 4.0 * c.B * K, s);
@@ -409,12 +426,101 @@ sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, flo
     for (int i = c.n1; i < c.n1 + c.n2; ++i)
       if ((st = run_block(h, xs, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
   }
-  // stage 3: dense late
   for (int i = c.n1 + c.n2; i < N; ++i)
     if ((st = run_block(h, xs, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
+  return SR_OK;
+}
+
+}  // namespace
+
+sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, float keep_ratio,
+                     uint64_t seed, void* out, int32_t* idx_out, void* stream) {
+  int32_t K = 0;
+  sr_status st = check_forward_args(h, x, w, keep_ratio, out, &K);
+  if (st != SR_OK) return st;
+  if (idx_out && !aligned(idx_out, 4)) return fail(SR_ERR_INVALID_ARG, "idx_out misaligned");
+  if (idx_out && K < 1) return fail(SR_ERR_INVALID_ARG, "K = floor(L * keep_ratio) is 0");
+  const sr_config& c = h->cfg;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t n = size_t(c.B) * c.L * c.D;
+  float* xs = static_cast<float*>(h->at(h->plan.xs));
+  const sr::PdlScope pdl(false);             // the widen waits for whatever came before
+  if ((st = widen_and_early(h, x, w, xs, s)) != SR_OK) return st;
+  const sr::PdlScope pdl_rest(!h->trace);
+  if ((st = route_and_late(h, xs, w, keep_ratio, K, seed, idx_out, s)) != SR_OK) return st;
   {
-    TraceScope t(h, SR_KERN_COPY, 0.0, double(bytes) + 4.0 * n, s);
+    TraceScope t(h, SR_KERN_COPY, 0.0, double(n) * (h->es + 4.0), s);
     SR_CUDA(sr::launch_narrow(h->dt, xs, out, n, s), "narrow out");
+  }
+  return SR_OK;
+}
+
+size_t sr_ensemble_workspace_bytes(const sr_config* cfg) {
+  if (validate_config(cfg) != SR_OK) return 0;
+  // the dense-early result and the fp32 sum of the members
+  return 2 * align_up(size_t(cfg->B) * cfg->L * cfg->D * sizeof(float));
+}
+
+sr_status sr_forward_ensemble(sr_handle* h, const void* x, const sr_block_weights* w,
+                              float keep_ratio, const uint64_t* seeds, int32_t M,
+                              void* ens_workspace, size_t ens_ws_bytes, void* out,
+                              void* members_out, int32_t* idx_out, void* stream) {
+  int32_t K = 0;
+  sr_status st = check_forward_args(h, x, w, keep_ratio, out, &K);
+  if (st != SR_OK) return st;
+  if (M < 1 || !seeds) return fail(SR_ERR_INVALID_ARG, "need M >= 1 seeds");
+  const sr_config& c = h->cfg;
+  const size_t n = size_t(c.B) * c.L * c.D;
+  const size_t fbytes = align_up(n * sizeof(float));
+  if (!ens_workspace || !aligned(ens_workspace, kAlign) || ens_ws_bytes < 2 * fbytes)
+    return fail(SR_ERR_WORKSPACE, "ensemble workspace NULL, misaligned or too small");
+  if (members_out && !aligned(members_out, 16))
+    return fail(SR_ERR_INVALID_ARG, "members_out must be 16-byte aligned");
+  if (idx_out && (!aligned(idx_out, 4) || K < 1))
+    return fail(SR_ERR_INVALID_ARG, "idx_out misaligned or K = 0");
+  const size_t bytes = n * h->es;
+  if (members_out) {
+    // members_out must not overlap x or out
+    const char* mb = static_cast<const char*>(members_out);
+    const char* xb = static_cast<const char*>(x);
+    const char* ob = static_cast<const char*>(out);
+    const size_t mbytes = size_t(M) * bytes;
+    if ((mb < xb + bytes && xb < mb + mbytes) || (mb < ob + bytes && ob < mb + mbytes))
+      return fail(SR_ERR_INVALID_ARG, "members_out overlaps x or out");
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  float* xs = static_cast<float*>(h->at(h->plan.xs));
+  float* xe = static_cast<float*>(ens_workspace);
+  float* acc = reinterpret_cast<float*>(static_cast<char*>(ens_workspace) + fbytes);
+  const sr::PdlScope pdl(false);
+  // the dense-early blocks do not depend on the seed: once for all members
+  if ((st = widen_and_early(h, x, w, xs, s)) != SR_OK) return st;
+  const sr::PdlScope pdl_rest(!h->trace);
+  if (M > 1) {
+    TraceScope t(h, SR_KERN_COPY, 0.0, 8.0 * n, s);
+    SR_CUDA(sr::launch_accumulate(xs, xe, n, true, s), "keep the dense-early result");
+  }
+  for (int32_t m = 0; m < M; ++m) {
+    if (m > 0) {
+      TraceScope t(h, SR_KERN_COPY, 0.0, 8.0 * n, s);
+      SR_CUDA(sr::launch_accumulate(xe, xs, n, true, s), "restore the dense-early result");
+    }
+    int32_t* idx_m = idx_out ? idx_out + size_t(m) * c.B * K : nullptr;
+    if ((st = route_and_late(h, xs, w, keep_ratio, K, seeds[m], idx_m, s)) != SR_OK) return st;
+    if (members_out) {
+      TraceScope t(h, SR_KERN_COPY, 0.0, double(n) * (h->es + 4.0), s);
+      SR_CUDA(sr::launch_narrow(h->dt, xs, static_cast<char*>(members_out) + size_t(m) * bytes, n, s),
+              "narrow member");
+    }
+    if (M > 1) {
+      TraceScope t(h, SR_KERN_COPY, 0.0, (m == 0 ? 8.0 : 12.0) * n, s);
+      SR_CUDA(sr::launch_accumulate(xs, acc, n, m == 0, s), "sum of the members");
+    }
+  }
+  {
+    // the mean of the members' fp32 results, rounded once
+    TraceScope t(h, SR_KERN_COPY, 0.0, double(n) * (h->es + 4.0), s);
+    SR_CUDA(sr::launch_narrow(h->dt, M > 1 ? acc : xs, out, n, s, 1.0f / float(M)), "narrow mean");
   }
   return SR_OK;
 }

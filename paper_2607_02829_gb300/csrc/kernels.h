@@ -72,7 +72,11 @@ cudaError_t launch_gather_rows(const float* x, const int32_t* idx, int B, int L,
 
 // ---- storage dtype <-> fp32 residual stream, n elements (n % 8 == 0) ------
 cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream_t s);
-cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStream_t s);
+// narrow rounds scale * x once to the storage dtype
+cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStream_t s,
+                          float scale = 1.0f);
+// acc = x (first) or acc += x, fp32, n % 4 == 0
+cudaError_t launch_accumulate(const float* x, float* acc, size_t n, bool first, cudaStream_t s);
 
 // ---- LayerNorm over D from the fp32 stream into the storage dtype ---------
 //      y = (x - mean) / sqrt(var + eps) * g + b

@@ -119,9 +119,27 @@ widen_kernel(const T* __restrict__ x, float* __restrict__ y, size_t nvec) {
   }
 }
 
+// acc = x (first) or acc += x over the fp32 stream, 4-float vectors
+__global__ void __launch_bounds__(256)
+accumulate_kernel(const float* __restrict__ x, float* __restrict__ acc, size_t nvec, int first) {
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
+  const float4* xv = reinterpret_cast<const float4*>(x);
+  float4* av = reinterpret_cast<float4*>(acc);
+  for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
+       i += size_t(gridDim.x) * blockDim.x) {
+    float4 v = __ldg(xv + i);
+    if (!first) {
+      const float4 a = av[i];
+      v = make_float4(a.x + v.x, a.y + v.y, a.z + v.z, a.w + v.w);
+    }
+    av[i] = v;
+  }
+}
+
 template <typename T>
 __global__ void __launch_bounds__(256)
-narrow_kernel(const float* __restrict__ x, T* __restrict__ y, size_t nvec) {
+narrow_kernel(const float* __restrict__ x, T* __restrict__ y, size_t nvec, float scale) {
   pdl_wait();      // the previous kernel's writes are visible from here
   pdl_trigger();
   constexpr int V = Elem<T>::kVec;
@@ -132,7 +150,8 @@ narrow_kernel(const float* __restrict__ x, T* __restrict__ y, size_t nvec) {
 #pragma unroll
     for (int q = 0; q < V / 4; ++q) {
       const float4 v4 = __ldg(in + q);
-      f[4 * q] = v4.x; f[4 * q + 1] = v4.y; f[4 * q + 2] = v4.z; f[4 * q + 3] = v4.w;
+      f[4 * q] = v4.x * scale; f[4 * q + 1] = v4.y * scale;
+      f[4 * q + 2] = v4.z * scale; f[4 * q + 3] = v4.w * scale;
     }
     reinterpret_cast<uint4*>(y)[i] = pack16(f);
   }
@@ -178,15 +197,21 @@ cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream
                   static_cast<const float*>(x), y, nvec);
 }
 
-cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStream_t s) {
+cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStream_t s, float scale) {
   if (dt == DType::BF16) {
     const size_t nvec = n / 8;
     return launch_k(narrow_kernel<bf16>, dim3(grid_for(nvec)), dim3(256), 0, s, 1, x,
-                    static_cast<bf16*>(y), nvec);
+                    static_cast<bf16*>(y), nvec, scale);
   }
   const size_t nvec = n / 4;
   return launch_k(narrow_kernel<float>, dim3(grid_for(nvec)), dim3(256), 0, s, 1, x,
-                  static_cast<float*>(y), nvec);
+                  static_cast<float*>(y), nvec, scale);
+}
+
+cudaError_t launch_accumulate(const float* x, float* acc, size_t n, bool first, cudaStream_t s) {
+  const size_t nvec = n / 4;
+  return launch_k(accumulate_kernel, dim3(grid_for(nvec)), dim3(256), 0, s, 1, x, acc, nvec,
+                  first ? 1 : 0);
 }
 
 cudaError_t launch_layernorm(DType dt, const float* x, const void* g, const void* b, void* y,

@@ -124,3 +124,39 @@ def test_routed_only_workspace_is_smaller_and_rejects_the_dense_path(L):
         assert e.value.status == b.SR_ERR_WORKSPACE
     finally:
         b.sr_destroy(h)
+
+
+def test_ensemble_workspace_and_argument_errors(L):
+    from paper_2607_02829_gb300 import binding as b
+    cfg = b.make_config(2, 512, 256, 4, 1, 2, 1, dtype="f32")
+    ens = b.sr_ensemble_workspace_bytes(cfg)
+    assert ens >= 2 * 2 * 512 * 256 * 4
+    bad = b.make_config(2, 512, 250, 4, 1, 2, 1, dtype="f32")
+    assert b.sr_ensemble_workspace_bytes(bad) == 0
+    h = _handle(b, cfg, b.sr_workspace_bytes(cfg, 0.25))
+    try:
+        w = (b.sr_block_weights * 4)()
+        for i in range(4):
+            for f in b.WEIGHT_FIELDS:
+                setattr(w[i], f, 0x200000)
+        X, O, E = 0x400000, 0x800000, 0x1000000
+        with pytest.raises(b.SRError) as e:          # no seeds
+            b.sr_forward_ensemble(h, X, w, 0.25, [], E, ens, O, None, None, None)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+        with pytest.raises(b.SRError) as e:          # no ensemble workspace
+            b.sr_forward_ensemble(h, X, w, 0.25, [1, 2], 0, ens, O, None, None, None)
+        assert e.value.status == b.SR_ERR_WORKSPACE
+        with pytest.raises(b.SRError) as e:          # short ensemble workspace
+            b.sr_forward_ensemble(h, X, w, 0.25, [1, 2], E, ens - 256, O, None, None, None)
+        assert e.value.status == b.SR_ERR_WORKSPACE
+        with pytest.raises(b.SRError) as e:          # misaligned ensemble workspace
+            b.sr_forward_ensemble(h, X, w, 0.25, [1, 2], E + 16, ens, O, None, None, None)
+        assert e.value.status == b.SR_ERR_WORKSPACE
+        with pytest.raises(b.SRError) as e:          # keep ratio out of range
+            b.sr_forward_ensemble(h, X, w, 1.5, [1, 2], E, ens, O, None, None, None)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+        with pytest.raises(b.SRError) as e:          # members_out overlapping out
+            b.sr_forward_ensemble(h, X, w, 0.25, [1, 2], E, ens, O, O + 4096, None, None)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+    finally:
+        b.sr_destroy(h)

@@ -171,3 +171,34 @@ def test_forward_parity_topk_selector_small():
     assert err <= TOL["bf16"], err
     x0, _ = gpu_forward(wl, x, ws, n_split=(1, 0, 0), want_idx=False)
     assert np.array_equal(idx, o.select_topk_l2(synth.stored_as_f64(x0), 64))
+
+
+# ------------------------------------------------------------ implicit ensemble
+@pytest.mark.parametrize("dtype,split,r", [("bf16", (1, 2, 1), 0.25), ("f32", (1, 2, 1), 0.5),
+                                            ("bf16", (2, 1, 0), 0.25), ("bf16", (1, 2, 1), 1.0)])
+def test_ensemble_members_bitwise_and_mean(dtype, split, r):
+    from paper_2607_02829_gb300 import binding as b
+    wl = _tiny(dtype, B=2, L=200, heads=2, split=split, r=r)
+    x, ws = synth.make_inputs(wl)
+    seeds = [3, 77, 2**63 + 5]
+    n1, n2, n3 = split
+    cfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, n1, n2, n3, dtype=dtype)
+    enc = b.Encoder(cfg, max_keep_ratio=r)
+    xd = x.cuda()
+    wd = [{k: v.cuda() for k, v in blk.items()} for blk in ws[:n1 + n2 + n3]]
+    warr = b.weights_array(wd)
+    mean, members, idx = enc.forward_ensemble(xd, warr, r, seeds, want_members=True, want_idx=r < 1.0)
+    for m, s in enumerate(seeds):
+        y, i1 = enc.forward(xd, warr, r, s, want_idx=r < 1.0)
+        assert torch.equal(members[m], y)          # member m is exactly sr_forward(seed m)
+        if r < 1.0:
+            assert torch.equal(idx[m], i1)
+    torch.cuda.synchronize()
+    ref, _, ridx = o.forward_ensemble(synth.stored_as_f64(x), o.as_f64_weights(ws[:n1 + n2 + n3]),
+                                      n1, n2, n3, wl.heads, r, seeds, threads=8)
+    if r < 1.0:
+        for m in range(len(seeds)):
+            assert np.array_equal(idx[m].cpu().numpy(), ridx[m])
+    err = max_norm_rel(synth.stored_as_f64(mean.cpu()), ref)
+    assert err <= TOL[dtype], err
+    enc.close()

@@ -301,3 +301,43 @@ def test_topk_selector_in_forward_uses_post_dense_state():
     out, idx, x0 = o.forward(x, ws, 1, 1, 1, heads=2, keep_ratio=0.25, selector="topk_l2",
                              return_stages=True)
     assert np.array_equal(idx, o.select_topk_l2(x0, 6))
+
+
+# ------------------------------------------------------------------ implicit ensemble
+def test_ensemble_of_the_dense_path_is_the_dense_stack():
+    # r = 1 routes nothing, so every member is the dense stack and their mean
+    # (four equal terms, an exact division by 4) is too
+    x, ws = _tiny_model()
+    mean, members, idxs = o.forward_ensemble(x, ws, 1, 2, 1, heads=2, keep_ratio=1.0,
+                                             seeds=[1, 2, 3, 4])
+    assert np.array_equal(mean, o.dense_stack(x, ws, heads=2))
+    assert all(i is None for i in idxs)
+
+
+def test_ensemble_members_and_mean():
+    x, ws = _tiny_model(N=3)
+    seeds = [5, 11, 2**64 - 3]
+    mean, members, idxs = o.forward_ensemble(x, ws, 1, 1, 1, heads=2, keep_ratio=0.25, seeds=seeds)
+    for s, y, idx in zip(seeds, members, idxs):
+        y1, idx1 = o.forward(x, ws, 1, 1, 1, heads=2, keep_ratio=0.25, seed=s)
+        assert np.array_equal(y, y1) and np.array_equal(idx, idx1)
+    assert np.allclose(mean, (members[0] + members[1] + members[2]) / 3.0, rtol=0, atol=1e-15)
+    assert not np.array_equal(idxs[0], idxs[1])
+
+
+def test_ensemble_passthrough_tokens():
+    # with no late blocks, a token no member selects keeps its pre-routing value
+    # exactly in the mean, and a token one of two members selects is the
+    # average of that member's value and the pre-routing value
+    x, ws = _tiny_model(N=2)
+    mean, members, idxs = o.forward_ensemble(x, ws, 1, 1, 0, heads=2, keep_ratio=0.25, seeds=[7, 8])
+    _, _, x0 = o.forward(x, ws, 1, 1, 0, heads=2, keep_ratio=0.25, seed=7, return_stages=True)
+    B, L, _ = x.shape
+    for b in range(B):
+        s0, s1 = set(idxs[0][b].tolist()), set(idxs[1][b].tolist())
+        for i in range(L):
+            if i not in s0 and i not in s1:
+                assert np.array_equal(mean[b, i], x0[b, i])
+            elif (i in s0) != (i in s1):
+                m = 0 if i in s0 else 1
+                assert np.allclose(mean[b, i], 0.5 * (members[m][b, i] + x0[b, i]), rtol=0, atol=1e-15)
