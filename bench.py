@@ -351,7 +351,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--split", default=None,
                     help="override the block split n1,n2,n3 (kernel studies and profiling)")
-    ap.add_argument("--sweep", choices=["gather", "ensemble"], default=None,
+    ap.add_argument("--sweep", choices=["gather", "ensemble", "cross_attention"], default=None,
                     help="size sweep of one kernel (prints one JSON line per size)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -366,6 +366,8 @@ def main():
         return gather_sweep(args)
     if args.sweep == "ensemble":
         return ensemble_sweep(args)
+    if args.sweep == "cross_attention":
+        return cross_attention_sweep(args)
 
     import torch
     import torch.distributed as dist
@@ -512,6 +514,46 @@ def ensemble_sweep(args):
                           "speedup_vs_separate": sep_ms / ens_ms,
                           "member_tokens_per_s": wl.B * wl.L * M / (ens_ms * 1e-3)}), flush=True)
     enc.close()
+
+
+def cross_attention_sweep(args):
+    """Asymmetric attention (queries from the routed tokens, keys/values from the
+    full sequence) at the 0.25 deg shapes, 16 heads: CUDA-event time per call
+    with L2 flushed before each, against the bf16 tensor peak."""
+    import torch
+    from paper_2607_02829_gb300 import binding as b, build
+    build.build()
+    peaks = _peaks()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    s = torch.cuda.current_stream()
+    heads = 16
+    D = 64 * heads
+    for (B, Tq, Tkv) in [(1, 4050, 16200), (1, 16200, 16200), (1, 2025, 16200), (8, 512, 2048)]:
+        q = torch.randn(B, Tq, D, device="cuda").to(torch.bfloat16)
+        kv = torch.randn(B, Tkv, 2 * D, device="cuda").to(torch.bfloat16)
+        out = torch.empty(B, Tq, D, dtype=torch.bfloat16, device="cuda")
+
+        def call():
+            b.sr_cross_attention(q.data_ptr(), kv.data_ptr(), B, Tq, Tkv, heads, out.data_ptr(),
+                                 None, s.cuda_stream)
+        for _ in range(args.warmup):
+            call()
+        tot = 0.0
+        for _ in range(args.steps):
+            flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(s)
+            call()
+            e1.record(s)
+            torch.cuda.synchronize()
+            tot += e0.elapsed_time(e1)
+        ms = tot / args.steps
+        tf = 4.0 * B * heads * Tq * Tkv * 64 / (ms * 1e-3) / 1e12
+        print(json.dumps({"sweep": "cross_attention", "B": B, "Tq": Tq, "Tkv": Tkv, "heads": heads,
+                          "ms": ms, "tflops": tf,
+                          "frac_of_burst": tf / peaks["bf16_tflops"]}), flush=True)
+        del q, kv, out
 
 
 def run_reference(args, rank, world):

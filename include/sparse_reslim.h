@@ -148,6 +148,23 @@ sr_status sr_forward_ensemble(sr_handle* h, const void* x, const sr_block_weight
                               void* ens_workspace, size_t ens_ws_bytes, void* out,
                               void* members_out, int32_t* idx_out, void* stream);
 
+/* Asymmetric attention (Sec. 3.5, "Integration with generative forecasting";
+ * Alg. 2): queries from one token set, keys and values from another, within
+ * each sample and per head: out = softmax(q k^T / 8) v.  In the EDM model's
+ * sparse stage the K routed tokens attend over the full L-token conditioning
+ * sequence, O(K L D) instead of O(L^2 D).  Standalone: no handle.
+ *  q     : [B, Tq, D] bf16 device, head h in columns [64h, 64h + 64).
+ *  kv    : [B, Tkv, 2D] bf16 device: k in columns [0, D), v in [D, 2D).
+ *  out   : [B, Tq, D] bf16 device; must not overlap q or kv.
+ *  fault : optional device uint32 word; a wait of the kernel that runs out
+ *          sets its bit 0 (as sr_device_fault reports for the encoder).  NULL
+ *          to ignore.
+ * D = 64 * heads (heads 1..32); q, kv and out 16-byte aligned.  Host-checked
+ * errors: SR_ERR_INVALID_ARG (NULL or misaligned pointers, sizes below 1,
+ * overlap), SR_ERR_UNSUPPORTED (heads out of range or sizes past 2^31 elements). */
+sr_status sr_cross_attention(const void* q, const void* kv, int32_t B, int32_t Tq, int32_t Tkv,
+                             int32_t heads, void* out, uint32_t* fault, void* stream);
+
 /* sr_forward from and to HOST memory: copies x_host ([B, L, D], preferably
  * pinned) into the caller's device buffer `dev_xout`, runs sr_forward in place
  * on it, and copies the result back into out_host.  All three steps are

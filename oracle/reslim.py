@@ -163,6 +163,32 @@ def attention(qkv: np.ndarray, heads: int, pool: Optional[ThreadPoolExecutor] = 
     return out
 
 
+def cross_attention(q: np.ndarray, kv: np.ndarray, heads: int,
+                    pool: Optional[ThreadPoolExecutor] = None) -> np.ndarray:
+    """Asymmetric attention (Sec. 3.5, "Integration with generative
+    forecasting"; Alg. 2): queries from one token set, keys and values from
+    another, within each sample.  q: [B, Tq, D]; kv: [B, Tkv, 2D] with columns
+    [0, D) = k and [D, 2D) = v, head h owning columns [h dh, (h+1) dh) of each.
+    Returns [B, Tq, D]."""
+    B, Tq, D = q.shape
+    dh = D // heads
+    out = np.empty((B, Tq, D), dtype=np.float64)
+
+    def one(bh):
+        b, h = divmod(bh, heads)
+        c = slice(h * dh, (h + 1) * dh)
+        out[b, :, c] = _attention_one_head(np.ascontiguousarray(q[b][:, c]),
+                                           np.ascontiguousarray(kv[b, :, :D][:, c]),
+                                           np.ascontiguousarray(kv[b, :, D:][:, c]))
+
+    if pool is None:
+        for bh in range(B * heads):
+            one(bh)
+    else:
+        list(pool.map(one, range(B * heads)))
+    return out
+
+
 def block(x: np.ndarray, w: Dict[str, np.ndarray], heads: int, eps: float = 1e-5,
           pool: Optional[ThreadPoolExecutor] = None) -> np.ndarray:
     """One pre-LN ViT block on x [B, T, D] (Sec. 3.3 Eq. 11):

@@ -81,6 +81,8 @@ def lib() -> ctypes.CDLL:
                                           ctypes.POINTER(ctypes.c_uint64), i32, vp, sz, vp, vp, vp,
                                           vp]
         L.sr_forward_ensemble.restype = st
+        L.sr_cross_attention.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, vp]
+        L.sr_cross_attention.restype = st
         L.sr_destroy.argtypes = [vp]; L.sr_destroy.restype = st
         L.sr_trace_enable.argtypes = [vp, ctypes.c_int]; L.sr_trace_enable.restype = st
         L.sr_trace_read.argtypes = [vp, ctypes.POINTER(sr_trace_entry), ctypes.c_int]
@@ -149,6 +151,12 @@ def sr_forward_ensemble(handle: int, x: int, weights: ctypes.Array, keep_ratio: 
     _check(lib().sr_forward_ensemble(handle, x, weights, keep_ratio, arr, len(seeds), ens_ws,
                                      ens_ws_bytes, out, members_out, idx_out, stream),
            "sr_forward_ensemble")
+
+
+def sr_cross_attention(q: int, kv: int, B: int, Tq: int, Tkv: int, heads: int, out: int,
+                       fault: Optional[int], stream: int) -> None:
+    _check(lib().sr_cross_attention(q, kv, B, Tq, Tkv, heads, out, fault, stream),
+           "sr_cross_attention")
 
 
 def sr_destroy(handle: Optional[int]) -> None:

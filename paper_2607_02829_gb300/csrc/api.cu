@@ -525,6 +525,28 @@ sr_status sr_forward_ensemble(sr_handle* h, const void* x, const sr_block_weight
   return SR_OK;
 }
 
+sr_status sr_cross_attention(const void* q, const void* kv, int32_t B, int32_t Tq, int32_t Tkv,
+                             int32_t heads, void* out, uint32_t* fault, void* stream) {
+  if (!q || !kv || !out || !aligned(q, 16) || !aligned(kv, 16) || !aligned(out, 16))
+    return fail(SR_ERR_INVALID_ARG, "q, kv and out must be non-NULL and 16-byte aligned");
+  if (fault && !aligned(fault, 4)) return fail(SR_ERR_INVALID_ARG, "fault word misaligned");
+  if (B < 1 || Tq < 1 || Tkv < 1) return fail(SR_ERR_INVALID_ARG, "B, Tq and Tkv must be >= 1");
+  if (heads < 1 || heads > 32) return fail(SR_ERR_UNSUPPORTED, "heads must lie in 1..32");
+  const double D = 64.0 * heads;
+  if (double(B) * Tq * D >= 2147483647.0 || double(B) * Tkv * 2.0 * D >= 2147483647.0)
+    return fail(SR_ERR_UNSUPPORTED, "B * T * width exceeds 2^31 elements");
+  const size_t qbytes = size_t(B) * Tq * size_t(D) * 2, kvbytes = size_t(B) * Tkv * size_t(D) * 4;
+  const char* ob = static_cast<const char*>(out);
+  const char* qb = static_cast<const char*>(q);
+  const char* kb = static_cast<const char*>(kv);
+  if ((ob < qb + qbytes && qb < ob + qbytes) || (ob < kb + kvbytes && kb < ob + qbytes))
+    return fail(SR_ERR_INVALID_ARG, "out overlaps q or kv");
+  SR_CUDA(sr::launch_cross_attention_tc(q, kv, out, B, Tq, Tkv, heads, fault,
+                                        static_cast<cudaStream_t>(stream)),
+          "cross attention");
+  return SR_OK;
+}
+
 sr_status sr_forward_host(sr_handle* h, const void* x_host, const sr_block_weights* w,
                           float keep_ratio, uint64_t seed, void* dev_xout, void* out_host,
                           int32_t* idx_out, void* stream) {

@@ -72,8 +72,9 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ out, int T,
-                    int heads, unsigned int* fault) {
+attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKV,
+                    bf16* __restrict__ out, int Tq, int Tkv, int heads, int qcol0, int kcol0,
+                    int vcol0, unsigned int* fault) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -83,13 +84,13 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
   AttSmem* sm = reinterpret_cast<AttSmem*>(sV + kStages * kTileBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qblocks = (T + kBQ - 1) / kBQ;
+  const int qblocks = (Tq + kBQ - 1) / kBQ;
   const int bh = blockIdx.x / qblocks;
   const int qb = blockIdx.x % qblocks;
   const int b = bh / heads, h = bh % heads;
   const int D = heads * kDh;
   const int q0 = qb * kBQ;
-  const int nkv = (T + kKV - 1) / kKV;
+  const int nkv = (Tkv + kKV - 1) / kKV;
 
   if (threadIdx.x == 0) {
     mbar_init(&sm->q_full, 1);
@@ -108,7 +109,10 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
     sm->abort = 0;
     fence_mbar_init();
   }
-  if (warp == 0 && lane == 0) prefetch_tmap(&tm);
+  if (warp == 0 && lane == 0) {
+    prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmKV);
+  }
   if (warp == 1) tmem_alloc(&sm->tmem_base, kTmemCols);
   tc_fence_before();
   __syncthreads();
@@ -129,8 +133,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
       if (lane == 0) {
         mbar_arrive_expect_tx(&sm->q_full, kQTiles * kTileBytes);
         for (int t = 0; t < kQTiles; ++t)
-          tma_load_3d(&tm, sQ + t * kTileBytes, &sm->q_full, h * kDh, q0 + t * kQTile, b);
-        const int kcol = D + h * kDh, vcol = 2 * D + h * kDh;
+          tma_load_3d(&tmQ, sQ + t * kTileBytes, &sm->q_full, qcol0 + h * kDh, q0 + t * kQTile, b);
+        const int kcol = kcol0 + h * kDh, vcol = vcol0 + h * kDh;
         // stages holding a load, and the parity of the phase each last used
         uint32_t kissued = 0, vissued = 0, kpar = 0, vpar = 0;
         int st = 0;
@@ -139,13 +143,13 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
           // a K stage frees once both tiles' S MMAs of key tile j - kStages are done
           if (!mbar_wait(&sm->k_empty[st], ph ^ 1, abort, fault)) break;
           mbar_arrive_expect_tx(&sm->k_full[st], kTileBytes);
-          tma_load_3d(&tm, sK + st * kTileBytes, &sm->k_full[st], kcol, j * kKV, b);
+          tma_load_3d(&tmKV, sK + st * kTileBytes, &sm->k_full[st], kcol, j * kKV, b);
           kissued |= 1u << st;
           kpar = (kpar & ~(1u << st)) | (ph << st);
           // a V stage once both tiles' P V MMAs of that key tile are
           if (!mbar_wait(&sm->v_empty[st], ph ^ 1, abort, fault)) break;
           mbar_arrive_expect_tx(&sm->v_full[st], kTileBytes);
-          tma_load_3d(&tm, sV + st * kTileBytes, &sm->v_full[st], vcol, j * kKV, b);
+          tma_load_3d(&tmKV, sV + st * kTileBytes, &sm->v_full[st], vcol, j * kKV, b);
           vissued |= 1u << st;
           vpar = (vpar & ~(1u << st)) | (ph << st);
           if (++st == kStages) { st = 0; ph ^= 1; }
@@ -244,7 +248,7 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
       tmem_wait_ld();
       tc_fence_before();
       mbar_arrive(&sm->s_free[t]);                 // S may now be overwritten
-      const int valid = T - j * kKV;               // keys of this tile that exist
+      const int valid = Tkv - j * kKV;             // keys of this tile that exist
       if (valid < kKV) {
 #pragma unroll
         for (int i = 0; i < kKV; ++i)
@@ -339,9 +343,9 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tm, bf16* __restrict__ o
       tmem_ld32(tO + 32, o[1]);
       tmem_wait_ld();
       const int row = q0 + t * kQTile + r;
-      if (row < T) {
+      if (row < Tq) {
         const float inv = 1.f / l_run;
-        uint4* dst = reinterpret_cast<uint4*>(out + (size_t(b) * T + row) * D + h * kDh);
+        uint4* dst = reinterpret_cast<uint4*>(out + (size_t(b) * Tq + row) * D + h * kDh);
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           const uint32_t* q = &o[i / 4][(i % 4) * 8];
@@ -375,28 +379,29 @@ cudaError_t get_encoder() {
   return cudaSuccess;
 }
 
-}  // namespace
 
-cudaError_t launch_attention_tc(const void* qkv, void* out, int B, int T, int heads,
-                                unsigned int* fault, cudaStream_t s) {
+// 3-D bf16 tensor map over [B, T, C] (row-major), box 64 columns x 128 rows x 1
+cudaError_t make_map_btc(CUtensorMap* map, const void* ptr, int B, int T, uint64_t C) {
   cudaError_t e = get_encoder();
   if (e != cudaSuccess) return e;
-  const uint64_t D3 = uint64_t(3) * heads * kDh;
-  // [B, T, 3D] bf16, box: 64 columns x 128 tokens x 1 sample
-  CUtensorMap tm;
-  cuuint64_t dims[3] = {D3, uint64_t(T), uint64_t(B)};
-  cuuint64_t strides[2] = {D3 * 2, D3 * 2 * uint64_t(T)};
+  cuuint64_t dims[3] = {C, uint64_t(T), uint64_t(B)};
+  cuuint64_t strides[2] = {C * 2, C * 2 * uint64_t(T)};
   cuuint32_t box[3] = {kDh, kKV, 1};
   cuuint32_t estr[3] = {1, 1, 1};
-  CUresult r = g_encode(&tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(qkv), dims,
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims,
                         strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+cudaError_t launch(const CUtensorMap& tq, const CUtensorMap& tkv, void* out, int B, int Tq,
+                   int Tkv, int heads, int qcol0, int kcol0, int vcol0, unsigned int* fault,
+                   cudaStream_t s) {
   static bool attr_set = false;
   if (!attr_set) {
     cudaFuncAttributes fa;
-    e = cudaFuncGetAttributes(&fa, attention_tc_kernel);
+    cudaError_t e = cudaFuncGetAttributes(&fa, attention_tc_kernel);
     if (e != cudaSuccess) return e;
     if (fa.numRegs < 168) return cudaErrorInvalidConfiguration;   // the register split needs 168
     e = cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -404,9 +409,31 @@ cudaError_t launch_attention_tc(const void* qkv, void* out, int B, int T, int he
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  const int grid = B * heads * ((T + kBQ - 1) / kBQ);
-  return launch_k(attention_tc_kernel, dim3(grid), dim3(kThreads), kSmemBytes, s, 1, tm,
-                  static_cast<bf16*>(out), T, heads, fault);
+  const int grid = B * heads * ((Tq + kBQ - 1) / kBQ);
+  return launch_k(attention_tc_kernel, dim3(grid), dim3(kThreads), kSmemBytes, s, 1, tq, tkv,
+                  static_cast<bf16*>(out), Tq, Tkv, heads, qcol0, kcol0, vcol0, fault);
+}
+
+}  // namespace
+
+cudaError_t launch_attention_tc(const void* qkv, void* out, int B, int T, int heads,
+                                unsigned int* fault, cudaStream_t s) {
+  const int D = heads * kDh;
+  CUtensorMap tm;
+  cudaError_t e = make_map_btc(&tm, qkv, B, T, uint64_t(3) * D);   // [B, T, 3D]: q | k | v
+  if (e != cudaSuccess) return e;
+  return launch(tm, tm, out, B, T, T, heads, 0, D, 2 * D, fault, s);
+}
+
+cudaError_t launch_cross_attention_tc(const void* q, const void* kv, void* out, int B, int Tq,
+                                      int Tkv, int heads, unsigned int* fault, cudaStream_t s) {
+  const int D = heads * kDh;
+  CUtensorMap tq, tkv;
+  cudaError_t e = make_map_btc(&tq, q, B, Tq, uint64_t(D));        // [B, Tq, D]
+  if (e != cudaSuccess) return e;
+  e = make_map_btc(&tkv, kv, B, Tkv, uint64_t(2) * D);             // [B, Tkv, 2D]: k | v
+  if (e != cudaSuccess) return e;
+  return launch(tq, tkv, out, B, Tq, Tkv, heads, 0, 0, D, fault, s);
 }
 
 }  // namespace sr

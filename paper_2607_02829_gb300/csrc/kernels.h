@@ -118,5 +118,9 @@ cudaError_t launch_attention_simt(DType dt, const void* qkv, void* out, int B, i
                                   cudaStream_t s);
 cudaError_t launch_attention_tc(const void* qkv, void* out, int B, int T, int heads,
                                 unsigned int* fault, cudaStream_t s);
+// Queries and keys/values from different token sets: q [B*Tq, D], kv [B*Tkv, 2D]
+// (k | v), out [B*Tq, D]; the same kernel with two tensor maps (bf16).
+cudaError_t launch_cross_attention_tc(const void* q, const void* kv, void* out, int B, int Tq,
+                                      int Tkv, int heads, unsigned int* fault, cudaStream_t s);
 
 }  // namespace sr

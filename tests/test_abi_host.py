@@ -160,3 +160,22 @@ def test_ensemble_workspace_and_argument_errors(L):
         assert e.value.status == b.SR_ERR_INVALID_ARG
     finally:
         b.sr_destroy(h)
+
+
+def test_cross_attention_argument_errors(L):
+    from paper_2607_02829_gb300 import binding as b
+    Q, KV, O = 0x400000, 0x800000, 0x2000000
+    cases = [
+        (dict(q=0), b.SR_ERR_INVALID_ARG), (dict(out=O + 8), b.SR_ERR_INVALID_ARG),
+        (dict(B=0), b.SR_ERR_INVALID_ARG), (dict(Tq=0), b.SR_ERR_INVALID_ARG),
+        (dict(Tkv=0), b.SR_ERR_INVALID_ARG), (dict(heads=0), b.SR_ERR_UNSUPPORTED),
+        (dict(heads=33), b.SR_ERR_UNSUPPORTED), (dict(out=Q + 64), b.SR_ERR_INVALID_ARG),
+        (dict(Tkv=1 << 22), b.SR_ERR_UNSUPPORTED),
+    ]
+    for kw, status in cases:
+        a = dict(q=Q, kv=KV, B=2, Tq=100, Tkv=300, heads=2, out=O, fault=None, stream=None)
+        a.update(kw)
+        with pytest.raises(b.SRError) as e:
+            b.sr_cross_attention(a["q"], a["kv"], a["B"], a["Tq"], a["Tkv"], a["heads"], a["out"],
+                                 a["fault"], a["stream"])
+        assert e.value.status == status, kw

@@ -202,3 +202,47 @@ def test_ensemble_members_bitwise_and_mean(dtype, split, r):
     err = max_norm_rel(synth.stored_as_f64(mean.cpu()), ref)
     assert err <= TOL[dtype], err
     enc.close()
+
+
+# ------------------------------------------------------------ asymmetric attention
+@pytest.mark.parametrize("B,Tq,Tkv,heads", [(2, 300, 1000, 2), (1, 129, 77, 1), (3, 1, 5, 4),
+                                            (1, 257, 256, 2), (2, 64, 1, 1)])
+def test_cross_attention_parity(B, Tq, Tkv, heads):
+    from paper_2607_02829_gb300 import binding as b
+    D = 64 * heads
+    g = torch.Generator().manual_seed(B * 1000 + Tq + Tkv)
+    q = torch.randn(B, Tq, D, generator=g).to(torch.bfloat16)
+    kv = torch.randn(B, Tkv, 2 * D, generator=g).to(torch.bfloat16)
+    out = torch.empty(B, Tq, D, dtype=torch.bfloat16, device="cuda")
+    fault = torch.zeros(1, dtype=torch.int32, device="cuda")
+    qd, kvd = q.cuda(), kv.cuda()
+    b.sr_cross_attention(qd.data_ptr(), kvd.data_ptr(), B, Tq, Tkv, heads, out.data_ptr(),
+                         fault.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    assert int(fault.item()) == 0
+    ref = o.cross_attention(synth.stored_as_f64(q), synth.stored_as_f64(kv), heads)
+    err = max_norm_rel(synth.stored_as_f64(out.cpu()), ref)
+    assert err <= TOL["bf16"], err
+
+
+def test_cross_attention_routed_over_full_sequence_sampled():
+    # the 0.25 deg shape of the EDM sparse stage: 4050 routed queries over the
+    # 16200-token conditioning sequence, 16 heads; the oracle on sampled rows
+    from paper_2607_02829_gb300 import binding as b
+    B, Tq, Tkv, heads = 1, 4050, 16200, 16
+    D = 64 * heads
+    g = torch.Generator().manual_seed(4050)
+    q = torch.randn(B, Tq, D, generator=g).to(torch.bfloat16)
+    kv = torch.randn(B, Tkv, 2 * D, generator=g).to(torch.bfloat16)
+    out = torch.empty(B, Tq, D, dtype=torch.bfloat16, device="cuda")
+    fault = torch.zeros(1, dtype=torch.int32, device="cuda")
+    b.sr_cross_attention(q.cuda().data_ptr(), kv.cuda().data_ptr(), B, Tq, Tkv, heads,
+                         out.data_ptr(), fault.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    assert int(fault.item()) == 0
+    rows = np.random.default_rng(0).choice(Tq, 48, replace=False)
+    rows = np.concatenate([rows, [0, 255, 256, Tq - 1]])
+    ref = o.cross_attention(synth.stored_as_f64(q)[:, rows], synth.stored_as_f64(kv), heads)
+    got = synth.stored_as_f64(out.cpu())[:, rows]
+    err = max_norm_rel(got, ref)
+    assert err <= TOL["bf16"], err

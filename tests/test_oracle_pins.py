@@ -341,3 +341,45 @@ def test_ensemble_passthrough_tokens():
             elif (i in s0) != (i in s1):
                 m = 0 if i in s0 else 1
                 assert np.allclose(mean[b, i], 0.5 * (members[m][b, i] + x0[b, i]), rtol=0, atol=1e-15)
+
+
+# ------------------------------------------------------------------ asymmetric attention
+def test_cross_attention_against_torch_sdpa_and_bruteforce():
+    # queries and keys/values of different lengths (Sec. 3.5: Q from the K routed
+    # tokens, K and V from the L-token conditioning sequence)
+    rng = np.random.default_rng(5)
+    B, Tq, Tkv, H, dh = 2, 7, 13, 3, 8
+    D = H * dh
+    q = rng.standard_normal((B, Tq, D))
+    kv = rng.standard_normal((B, Tkv, 2 * D))
+    out = o.cross_attention(q, kv, H)
+    tq = torch.from_numpy(q).reshape(B, Tq, H, dh).transpose(1, 2)
+    tk = torch.from_numpy(kv[..., :D]).reshape(B, Tkv, H, dh).transpose(1, 2)
+    tv = torch.from_numpy(kv[..., D:]).reshape(B, Tkv, H, dh).transpose(1, 2)
+    ref = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv).transpose(1, 2).reshape(B, Tq, D)
+    assert np.allclose(out, ref.numpy(), rtol=0, atol=1e-13)
+    b, h, t, c = 1, 2, 6, 3
+    s = [sum(q[b, t, h * dh + j] * kv[b, u, h * dh + j] for j in range(dh)) / math.sqrt(dh)
+         for u in range(Tkv)]
+    m = max(s)
+    e = [math.exp(v_ - m) for v_ in s]
+    val = sum(e[u] * kv[b, u, D + h * dh + c] for u in range(Tkv)) / sum(e)
+    assert abs(out[b, t, h * dh + c] - val) < 1e-13
+
+
+def test_cross_attention_on_the_same_tokens_is_self_attention():
+    rng = np.random.default_rng(6)
+    B, T, H, dh = 2, 11, 2, 8
+    D = H * dh
+    qkv = rng.standard_normal((B, T, 3 * D))
+    assert np.array_equal(o.cross_attention(qkv[..., :D], qkv[..., D:], H), o.attention(qkv, H))
+
+
+def test_cross_attention_single_key_returns_its_value():
+    rng = np.random.default_rng(7)
+    B, Tq, H, dh = 2, 5, 2, 8
+    D = H * dh
+    q = rng.standard_normal((B, Tq, D))
+    kv = rng.standard_normal((B, 1, 2 * D))
+    out = o.cross_attention(q, kv, H)
+    assert np.allclose(out, np.broadcast_to(kv[:, :, D:], out.shape), rtol=0, atol=1e-15)
