@@ -29,10 +29,10 @@ L2_FLUSH_BYTES = 512 << 20          # > 129 MB of L2
 
 # DRAM bytes (read + write) per launch of a kernel kind on a workload, from one
 # ncu capture of the current kernel (profiles/attention_tc_c4_*.md): the 0.25 deg
-# forward runs 8 dense attention launches (114.35 MB each) and 16 sparse ones
-# (24.93 MB each).  None when no capture of the current kernel exists.
+# forward runs 8 dense attention launches (113.96 MB each) and 16 sparse ones
+# (24.94 MB each).  None when no capture of the current kernel exists.
 DRAM_TRAFFIC_PER_LAUNCH = {
-    ("attention", "c4_0p25deg_bf16"): (8 * 114.35e6 + 16 * 24.93e6) / 24,
+    ("attention", "c4_0p25deg_bf16"): (8 * 113.96e6 + 16 * 24.94e6) / 24,
 }
 
 
@@ -428,9 +428,11 @@ def main():
 
 
 def gather_sweep(args):
-    """Gather GB/s from 33 MB to 530 MB moved: one sparse block (split 0,1,0) of the
-    0.25 deg model (L=16200, D=1024, r=0.25) at batch 1..16, L2 flushed before
-    every traced forward; the gather kernel's CUDA-event time from the trace."""
+    """Gather GB/s from 33 MB to 530 MB of selected rows: one sparse block (split
+    0,1,0) of the 0.25 deg model (L=16200, D=1024, r=0.25) at batch 1..16, L2
+    flushed before every traced forward.  The gather of Eq. 8 runs fused with
+    the first sparse block's LN1; its CUDA-event time and algorithmic bytes
+    (selected rows read, h0 and LN1 written, index set) come from the trace."""
     import torch
     from paper_2607_02829_gb300 import binding as b, build, synth
     build.build()

@@ -184,7 +184,8 @@ sr_status sr_forward_host(sr_handle* h, const void* x_host, const sr_block_weigh
 typedef enum {
   SR_KERN_COPY = 0,          /* x -> out device copy when out != x */
   SR_KERN_SELECT = 1,        /* token selection (and the norms of the top-K selector) */
-  SR_KERN_GATHER = 2,        /* h0 = x[:, I, :] */
+  SR_KERN_GATHER = 2,        /* h0 = x[:, I, :] (Eq. 8), fused with LN1 of the first
+                                sparse block: reads the selected rows, writes h0 and LN1 */
   SR_KERN_LAYERNORM = 3,
   SR_KERN_GEMM_QKV = 4,      /* LN1(x) Wqkv^T + bqkv */
   SR_KERN_ATTENTION = 5,     /* softmax(q k^T / 8) v per (sample, head) */

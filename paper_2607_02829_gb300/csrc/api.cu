@@ -201,10 +201,12 @@ cudaError_t attention(const sr_handle* h, const void* qkv, void* out, int B, int
 // One pre-LN block (Sec. 3.3 Eq. 11) on the fp32 residual stream x [B*T, D], in
 // place.  With `scatter` set this is the last sparse block: its FC2 epilogue
 // writes x0 + (h_out - h0) into the rows idx of the stream `scatter_out`
-// [B*Lx, D] instead of x.
+// [B*Lx, D] instead of x.  With `gather_from` set this is the first sparse
+// block: its LN1 reads the rows idx of the stream `gather_from` [B*Lx, D]
+// directly and also writes them to x (the gather of Eq. 8, fused).
 sr_status run_block(const sr_handle* hd, float* x, int B, int T, const sr_block_weights& w,
                     bool scatter, float* scatter_out, const int32_t* idx, int Lx,
-                    cudaStream_t s) {
+                    cudaStream_t s, const float* gather_from = nullptr) {
   const sr_config& c = hd->cfg;
   const int rows = B * T, D = c.D, H = c.mlp_hidden;
   const double es = double(hd->es), R = double(rows);
@@ -213,7 +215,13 @@ sr_status run_block(const sr_handle* hd, float* x, int B, int T, const sr_block_
   void* att = hd->at(hd->plan.att);
   void* u = hd->at(hd->plan.u);
   const double ln_bytes = R * D * (4.0 + es) + 2.0 * D * es;
-  {
+  if (gather_from) {
+    // reads the selected rows, writes LN1 and the fp32 copy h0, plus the index set
+    TraceScope t(hd, SR_KERN_GATHER, 0.0, R * D * (8.0 + es) + 4.0 * R + 2.0 * D * es, s);
+    SR_CUDA(sr::launch_layernorm(hd->dt, gather_from, w.ln1_g, w.ln1_b, ln, rows, D, c.ln_eps, s,
+                                 idx, Lx, T, x),
+            "gather + layernorm1");
+  } else {
     TraceScope t(hd, SR_KERN_LAYERNORM, 0.0, ln_bytes, s);
     SR_CUDA(sr::launch_layernorm(hd->dt, x, w.ln1_g, w.ln1_b, ln, rows, D, c.ln_eps, s), "layernorm1");
   }
@@ -413,14 +421,13 @@ sr_status route_and_late(sr_handle* h, float* xs, const sr_block_weights* w, flo
   if (route || idx_out)
     if ((st = do_select(h, xs, K, seed, idx, s)) != SR_OK) return st;
   if (route) {
+    // the gather of Eq. 8 is fused into the first sparse block's LN1
     float* hs = static_cast<float*>(h->at(h->plan.hs));
-    {
-      TraceScope t(h, SR_KERN_GATHER, 0.0, 8.0 * c.B * K * c.D + 4.0 * c.B * K, s);
-      SR_CUDA(sr::launch_gather_rows(xs, idx, c.B, c.L, K, c.D, hs, s), "gather");
-    }
     for (int i = c.n1; i < c.n1 + c.n2; ++i) {
       const bool last = i == c.n1 + c.n2 - 1;
-      if ((st = run_block(h, hs, c.B, K, w[i], last, xs, idx, c.L, s)) != SR_OK) return st;
+      if ((st = run_block(h, hs, c.B, K, w[i], last, xs, idx, c.L, s, i == c.n1 ? xs : nullptr)) !=
+          SR_OK)
+        return st;
     }
   } else {
     for (int i = c.n1; i < c.n1 + c.n2; ++i)

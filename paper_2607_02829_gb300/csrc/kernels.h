@@ -66,10 +66,6 @@ cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t*
 // Largest L the one-CTA-per-sample selection kernels accept (keys in shared memory).
 int select_max_L();
 
-// ---- gather (Eq. 8) on the fp32 stream: h[b*K + k, :] = x[b*L + idx[b*K + k], :]
-cudaError_t launch_gather_rows(const float* x, const int32_t* idx, int B, int L, int K, int D,
-                               float* h, cudaStream_t s);
-
 // ---- storage dtype <-> fp32 residual stream, n elements (n % 8 == 0) ------
 cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream_t s);
 // narrow rounds scale * x once to the storage dtype
@@ -80,8 +76,13 @@ cudaError_t launch_accumulate(const float* x, float* acc, size_t n, bool first, 
 
 // ---- LayerNorm over D from the fp32 stream into the storage dtype ---------
 //      y = (x - mean) / sqrt(var + eps) * g + b
+//      With idx set (LN1 of the first sparse block fused with the gather of
+//      Eq. 8): row r reads stream row (r / K) * L + idx[r] and also copies that
+//      fp32 row to hcopy[r].
 cudaError_t launch_layernorm(DType dt, const float* x, const void* g, const void* b, void* y,
-                             int rows, int D, float eps, cudaStream_t s);
+                             int rows, int D, float eps, cudaStream_t s,
+                             const int32_t* idx = nullptr, int L = 0, int K = 0,
+                             float* hcopy = nullptr);
 
 // ---- GEMM C = A B^T with fused epilogues ---------------------------------
 // A [M, K] row-major, B [N, K] row-major (nn.Linear weight), both in the storage

@@ -9,40 +9,19 @@
 namespace sr {
 namespace {
 
-// h[b*K + k, :] = x[b*L + idx[b*K + k], :]  -- a bit copy of D fp32 values.
-template <int NV>
-__global__ void __launch_bounds__(256)
-gather_rows_kernel(const float* __restrict__ x, const int32_t* __restrict__ idx, int L, int K,
-                   int D, int rows, float* __restrict__ h) {
-  pdl_wait();      // the previous kernel's writes are visible from here
-  pdl_trigger();
-  constexpr int V = 4;
-  const int lane = threadIdx.x & 31;
-  const int nv = D / V;
-  const int warps = (gridDim.x * blockDim.x) >> 5;
-  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += warps) {
-    const int b = r / K;
-    const int src = b * L + __ldg(idx + r);
-    const uint4* s = reinterpret_cast<const uint4*>(x + size_t(src) * D);
-    uint4* d = reinterpret_cast<uint4*>(h + size_t(r) * D);
-    uint4 v[NV];
-#pragma unroll
-    for (int j = 0; j < NV; ++j)
-      if (lane + 32 * j < nv) v[j] = __ldg(s + lane + 32 * j);
-#pragma unroll
-    for (int j = 0; j < NV; ++j)
-      if (lane + 32 * j < nv) d[lane + 32 * j] = v[j];
-  }
-}
-
 // y = (x - mean) / sqrt(var + eps) * g + b from the fp32 stream x into the
 // storage dtype T, statistics in fp32, two passes over the row held in
 // registers (biased variance).  Rows are read as 4-float vectors, g, b and y
 // move as 16-byte vectors of T.
+// With idx set, this is LN1 of the first sparse block fused with the gather
+// of Eq. 8: output row r (sample r / K) normalises stream row (r / K) * L +
+// idx[r], and that fp32 row is also copied to hcopy[r] (h0, the start of the
+// routed stream).
 template <typename T, int NV>
 __global__ void __launch_bounds__(256)
 layernorm_kernel(const float* __restrict__ x, const T* __restrict__ g, const T* __restrict__ bta,
-                 T* __restrict__ y, int rows, int D, float eps) {
+                 T* __restrict__ y, int rows, int D, float eps, const int32_t* __restrict__ idx,
+                 int L, int K, float* __restrict__ hcopy) {
   pdl_wait();      // the previous kernel's writes are visible from here
   pdl_trigger();
   constexpr int V = Elem<T>::kVec;
@@ -50,7 +29,8 @@ layernorm_kernel(const float* __restrict__ x, const T* __restrict__ g, const T* 
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   if (row >= rows) return;
   const int nv = D / V;
-  const float4* xr = reinterpret_cast<const float4*>(x + size_t(row) * D);
+  const size_t src = idx ? size_t(row / K) * L + size_t(__ldg(idx + row)) : size_t(row);
+  const float4* xr = reinterpret_cast<const float4*>(x + src * D);
   float f[NV][V];
   float sum = 0.f;
 #pragma unroll
@@ -76,6 +56,16 @@ layernorm_kernel(const float* __restrict__ x, const T* __restrict__ g, const T* 
     }
   }
   const float rstd = rsqrtf(warp_sum(sq) * inv_d + eps);
+  if (hcopy) {
+    float4* hr = reinterpret_cast<float4*>(hcopy + size_t(row) * D);
+#pragma unroll
+    for (int j = 0; j < NV; ++j)
+      if (lane + 32 * j < nv)
+#pragma unroll
+        for (int q = 0; q < V / 4; ++q)
+          hr[(lane + 32 * j) * (V / 4) + q] =
+              make_float4(f[j][4 * q], f[j][4 * q + 1], f[j][4 * q + 2], f[j][4 * q + 3]);
+  }
   const uint4* gr = reinterpret_cast<const uint4*>(g);
   const uint4* br = reinterpret_cast<const uint4*>(bta);
   uint4* yr = reinterpret_cast<uint4*>(y + size_t(row) * D);
@@ -91,15 +81,6 @@ layernorm_kernel(const float* __restrict__ x, const T* __restrict__ g, const T* 
       yr[v] = pack16(o);
     }
   }
-}
-
-template <int NV>
-cudaError_t gather_t(const float* x, const int32_t* idx, int B, int L, int K, int D, float* h,
-                     cudaStream_t s) {
-  const int rows = B * K;
-  int blocks = (rows + 7) / 8;
-  if (blocks > 152 * 16) blocks = 152 * 16;
-  return launch_k(gather_rows_kernel<NV>, dim3(blocks), dim3(256), 0, s, 1, x, idx, L, K, D, rows, h);
 }
 
 // Storage dtype <-> fp32 stream, n elements (n % 8 == 0), 16-byte vectors.
@@ -164,27 +145,16 @@ int grid_for(size_t nvec) {
 
 template <typename T, int NV>
 cudaError_t layernorm_t(const float* x, const void* g, const void* b, void* y, int rows, int D,
-                        float eps, cudaStream_t s) {
+                        float eps, cudaStream_t s, const int32_t* idx, int L, int K, float* hcopy) {
   return launch_k(layernorm_kernel<T, NV>, dim3((rows + 7) / 8), dim3(256), 0, s, 1, x,
                   static_cast<const T*>(g), static_cast<const T*>(b), static_cast<T*>(y), rows, D,
-                  eps);
+                  eps, idx, L, K, hcopy);
 }
 
 // vectors per lane needed for a row of D elements
 template <typename T> int lanes_nv(int D) { return (D / Elem<T>::kVec + 31) / 32; }
 
 }  // namespace
-
-cudaError_t launch_gather_rows(const float* x, const int32_t* idx, int B, int L, int K, int D,
-                               float* h, cudaStream_t s) {
-  const int nv = lanes_nv<float>(D);
-  if (nv <= 1) return gather_t<1>(x, idx, B, L, K, D, h, s);
-  if (nv <= 2) return gather_t<2>(x, idx, B, L, K, D, h, s);
-  if (nv <= 4) return gather_t<4>(x, idx, B, L, K, D, h, s);
-  if (nv <= 8) return gather_t<8>(x, idx, B, L, K, D, h, s);
-  if (nv <= 16) return gather_t<16>(x, idx, B, L, K, D, h, s);
-  return cudaErrorInvalidValue;
-}
 
 cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream_t s) {
   if (dt == DType::BF16) {
@@ -215,19 +185,20 @@ cudaError_t launch_accumulate(const float* x, float* acc, size_t n, bool first, 
 }
 
 cudaError_t launch_layernorm(DType dt, const float* x, const void* g, const void* b, void* y,
-                             int rows, int D, float eps, cudaStream_t s) {
+                             int rows, int D, float eps, cudaStream_t s, const int32_t* idx,
+                             int L, int K, float* hcopy) {
   if (dt == DType::BF16) {
     const int nv = lanes_nv<bf16>(D);
-    if (nv <= 1) return layernorm_t<bf16, 1>(x, g, b, y, rows, D, eps, s);
-    if (nv <= 2) return layernorm_t<bf16, 2>(x, g, b, y, rows, D, eps, s);
-    if (nv <= 4) return layernorm_t<bf16, 4>(x, g, b, y, rows, D, eps, s);
-    if (nv <= 8) return layernorm_t<bf16, 8>(x, g, b, y, rows, D, eps, s);
+    if (nv <= 1) return layernorm_t<bf16, 1>(x, g, b, y, rows, D, eps, s, idx, L, K, hcopy);
+    if (nv <= 2) return layernorm_t<bf16, 2>(x, g, b, y, rows, D, eps, s, idx, L, K, hcopy);
+    if (nv <= 4) return layernorm_t<bf16, 4>(x, g, b, y, rows, D, eps, s, idx, L, K, hcopy);
+    if (nv <= 8) return layernorm_t<bf16, 8>(x, g, b, y, rows, D, eps, s, idx, L, K, hcopy);
   } else {
     const int nv = lanes_nv<float>(D);
-    if (nv <= 1) return layernorm_t<float, 1>(x, g, b, y, rows, D, eps, s);
-    if (nv <= 2) return layernorm_t<float, 2>(x, g, b, y, rows, D, eps, s);
-    if (nv <= 4) return layernorm_t<float, 4>(x, g, b, y, rows, D, eps, s);
-    if (nv <= 8) return layernorm_t<float, 8>(x, g, b, y, rows, D, eps, s);
+    if (nv <= 1) return layernorm_t<float, 1>(x, g, b, y, rows, D, eps, s, idx, L, K, hcopy);
+    if (nv <= 2) return layernorm_t<float, 2>(x, g, b, y, rows, D, eps, s, idx, L, K, hcopy);
+    if (nv <= 4) return layernorm_t<float, 4>(x, g, b, y, rows, D, eps, s, idx, L, K, hcopy);
+    if (nv <= 8) return layernorm_t<float, 8>(x, g, b, y, rows, D, eps, s, idx, L, K, hcopy);
   }
   return cudaErrorInvalidValue;
 }
