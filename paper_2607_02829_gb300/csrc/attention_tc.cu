@@ -18,8 +18,9 @@
 //               an N = 64 MMA is 32 cycles of work, so the P V MMAs of each tile
 //               get their own issuing thread;
 //   warps 4-7   softmax of tile 0, warps 8-11 softmax of tile 1: one query row
-//               per thread.  Each reads its S row from TMEM, updates the
-//               running max and sum, computes P = 2^(s*c - m*c) as bf16 pairs
+//               per thread.  Each reads its S row from TMEM with the row
+//               maximum computed by the load itself (tcgen05.ld.red, sm_103a),
+//               updates the running max and sum, computes P = 2^(s*c - m*c) as bf16 pairs
 //               in registers and, once the previous P V has read the tile's P
 //               columns, writes them to tensor memory, where the P V MMA reads
 //               its A operand.
@@ -64,6 +65,21 @@ struct AttSmem {
 constexpr size_t kSmemBytes = 1024 /*align*/ + size_t(kQTiles) * kTileBytes +
                               size_t(kStages) * 2 * kTileBytes + 256;
 static_assert(sizeof(AttSmem) <= 256, "barrier block outgrew its reserve");
+
+// 32x32b.x32 TMEM load (as tmem_ld32) that also returns the maximum of the 32
+// values each thread receives (sm_103a: tcgen05.ld.red)
+__device__ __forceinline__ void tmem_ld32_max(uint32_t taddr, uint32_t (&r)[32], float& m) {
+  asm volatile(
+      "tcgen05.ld.red.sync.aligned.32x32b.x32.max.f32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10,"
+      " %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29,"
+      " %30, %31}, %32, [%33];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=f"(m)
+      : "r"(taddr));
+}
 
 __device__ __forceinline__ float max3(float a, float b, float c) {
   float d;
@@ -242,34 +258,26 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
       ok = __all_sync(0xffffffffu, mbar_wait(&sm->s_full[t], j & 1, abort, fault));
       if (!ok) break;
       tc_fence_after();
+      // S with its row maximum: the load reduces each thread's 32 columns
       uint32_t s[kKV / 32][32];
+      float pm[kKV / 32];
 #pragma unroll
-      for (int cc = 0; cc < kKV / 32; ++cc) tmem_ld32(tS + uint32_t(cc * 32), s[cc]);
+      for (int cc = 0; cc < kKV / 32; ++cc) tmem_ld32_max(tS + uint32_t(cc * 32), s[cc], pm[cc]);
       tmem_wait_ld();
       tc_fence_before();
       mbar_arrive(&sm->s_free[t]);                 // S may now be overwritten
+      float tmax = fmaxf(max3(pm[0], pm[1], pm[2]), pm[3]);
       const int valid = Tkv - j * kKV;             // keys of this tile that exist
       if (valid < kKV) {
+        // keys past the end are zero-filled (S = 0 there): mask them and take
+        // the maximum over the keys that exist
+        tmax = -INFINITY;
 #pragma unroll
-        for (int i = 0; i < kKV; ++i)
+        for (int i = 0; i < kKV; ++i) {
           if (i >= valid) s[i / 32][i % 32] = __float_as_uint(-INFINITY);
-      }
-      // row max: eight chains of three-input maxima
-      float pm[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) pm[k] = __uint_as_float(s[0][k]);
-#pragma unroll
-      for (int i = 8; i < kKV; i += 16) {
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          const int a = i + k, bb = i + 8 + k;
-          pm[k] = bb < kKV ? max3(pm[k], __uint_as_float(s[a / 32][a % 32]),
-                                  __uint_as_float(s[bb / 32][bb % 32]))
-                           : fmaxf(pm[k], __uint_as_float(s[a / 32][a % 32]));
+          tmax = fmaxf(tmax, __uint_as_float(s[i / 32][i % 32]));
         }
       }
-      const float tmax = max3(max3(pm[0], pm[1], pm[2]), max3(pm[3], pm[4], pm[5]),
-                              fmaxf(pm[6], pm[7]));
       float alpha = 1.f;
       bool rescale = false;
       if (j == 0) {
