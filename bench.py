@@ -29,10 +29,10 @@ L2_FLUSH_BYTES = 512 << 20          # > 129 MB of L2
 
 # DRAM bytes (read + write) per launch of a kernel kind on a workload, from one
 # ncu capture of the current kernel (profiles/attention_tc_c4_*.md): the 0.25 deg
-# forward runs 8 dense attention launches (113.96 MB each) and 16 sparse ones
-# (24.94 MB each).  None when no capture of the current kernel exists.
+# forward runs 8 dense attention launches (114.66 MB each) and 16 sparse ones
+# (24.93 MB each).  None when no capture of the current kernel exists.
 DRAM_TRAFFIC_PER_LAUNCH = {
-    ("attention", "c4_0p25deg_bf16"): (8 * 113.96e6 + 16 * 24.94e6) / 24,
+    ("attention", "c4_0p25deg_bf16"): (8 * 114.66e6 + 16 * 24.93e6) / 24,
 }
 
 
