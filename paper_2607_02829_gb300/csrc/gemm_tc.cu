@@ -36,14 +36,15 @@ struct GemmCfg {
   // each loads its own 128 rows of A and half of the tile's B rows
   static constexpr int kRowsTile = kPair ? 2 * BM : BM;
   static constexpr int kBRows = kPair ? BN / 2 : BN;
-  // the residual epilogue keeps two 32 x 32 fp32 residual tiles per epilogue
-  // warp in shared memory (64 KB), paid for with a shorter operand ring
-  static constexpr bool kTmaRes = E == Epi::BiasResidual && BN == 128;
+  // the residual epilogue of pair tiles keeps two 32 x 32 fp32 residual tiles
+  // per epilogue warp in shared memory (64 KB), paid for with a shorter operand
+  // ring on 256-column tiles
+  static constexpr bool kTmaRes = E == Epi::BiasResidual && kPair;
   // bf16 outputs of tiles at least 128 columns wide leave through TMA stores
   // from a 128-byte-swizzled 32 x 64 tile per epilogue warp (4 KB)
   static constexpr bool kTmaOut = (E == Epi::Bias || E == Epi::BiasGelu) && BN >= 128;
   static constexpr int kOutTileBytes = 32 * 128;
-  static constexpr int kStages = kPair ? 6 : (kTmaRes ? 4 : (BN == 256 ? 4 : 6));
+  static constexpr int kStages = kPair ? (kTmaRes && BN == 256 ? 5 : 6) : (BN == 256 ? 4 : 6);
   static constexpr int kABytes = BM * BK * 2;        // 16 KB
   static constexpr int kBBytes = kBRows * BK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
@@ -67,6 +68,7 @@ struct Smem {
 };
 static_assert(sizeof(Smem) <= 512, "the barrier block must fit its reserve in GemmCfg::kSmem");
 static_assert(GemmCfg<256, Epi::BiasResidual, true>::kSmem <= 232448, "pair config exceeds shared memory");
+static_assert(GemmCfg<256, Epi::Bias, true>::kSmem <= 232448, "pair config exceeds shared memory");
 
 // GELU(z) = z * Phi(z) with Phi from the erfc approximation of Abramowitz &
 // Stegun, Handbook of Mathematical Functions, formula 7.1.26 (absolute error
@@ -265,6 +267,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   tc_fence_after();
   const uint32_t tmem = sm->tmem_base;
   volatile int* abort = &sm->abort;
+  if (warp == 0 && lane == 0 && unit < tiles) {
+    // the weights do not depend on the previous kernel: the first tile's weight
+    // rows start moving into L2 while it finishes
+    const int brow = (unit % n_tiles) * BN + int(rank) * C::kBRows;
+    for (int kb = 0; kb < kblocks; ++kb) tma_prefetch_l2_2d(&tmB, kb * BK, brow);
+  }
   pdl_wait();      // the previous kernel's writes are visible from here
   pdl_trigger();
   // an abort in one CTA of a pair stops the other's waits too
@@ -413,35 +421,48 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                                lane);
         }
       } else if constexpr (C::kTmaRes) {
-        // residual tiles by TMA: both chunks of this warp (32 rows x 32 fp32, 128-byte
-        // swizzle) are requested before the accumulator is ready, updated in place
-        // and stored back by TMA
-        static_assert(BN == 128, "the TMA residual epilogue takes two 32-column chunks");
+        // residual tiles by TMA: the warp's half of the tile's columns is walked in
+        // 32-column chunks (32 rows x 32 fp32, 128-byte swizzle) through two
+        // buffers; the first two are requested before the accumulator is ready,
+        // each chunk is updated in place and stored back by TMA, and a buffer is
+        // refilled once its store has read it
+        constexpr int kChunks = BN / 64;
+        static_assert(kChunks % 2 == 0, "chunks alternate between two buffers");
         unsigned char* rbuf = reinterpret_cast<unsigned char*>(staging) +
                               size_t(warp - 2) * 2 * C::kResTileBytes;
         uint64_t* rbar = sm->res_full[warp - 2];
+        auto request = [&](int k) {   // lane 0 only
+          mbar_arrive_expect_tx(&rbar[k & 1], C::kResTileBytes);
+          tma_load_2d(&tmR, rbuf + (k & 1) * C::kResTileBytes, &rbar[k & 1],
+                      nt * BN + c_begin + 32 * k, row0);
+        };
+        // parity of chunk k's buffer barrier: each barrier completes kChunks / 2 times a tile
+        auto parity = [&](int k) { return uint32_t(it * (kChunks / 2) + (k >> 1)) & 1u; };
         if (lane == 0) {
-          bulk_wait_read_all();          // the previous tile's stores left these buffers
-#pragma unroll
-          for (int k = 0; k < 2; ++k) {
-            mbar_arrive_expect_tx(&rbar[k], C::kResTileBytes);
-            tma_load_2d(&tmR, rbuf + k * C::kResTileBytes, &rbar[k], nt * BN + c_begin + 32 * k, row0);
-          }
+          bulk_wait_read_all();          // the previous tile's stores left both buffers
+          request(0);
+          request(1);
+          // the later chunks move into L2 while the tile's mainloop runs: a launch
+          // whose tiles end together would otherwise stream the whole residual
+          // stream from HBM in its tail
+          if (row0 < M)
+            for (int k = 2; k < kChunks; ++k) tma_prefetch_l2_2d(&tmR, nt * BN + c_begin + 32 * k, row0);
         }
-        const uint32_t rph = uint32_t(it) & 1u;
+        int consumed = 0, requested = 2;
         bool ok = __all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault));
         if (ok) {
           tc_fence_after();
           const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
 #pragma unroll 1
-          for (int k = 0; k < 2 && ok; ++k) {
+          for (int k = 0; k < kChunks && ok; ++k) {
             const int c = c_begin + 32 * k;
             uint32_t r[32];
             tmem_ld32(tbase + uint32_t(c), r);
             tmem_wait_ld();
-            if (!(ok = __all_sync(0xffffffffu, mbar_wait(&rbar[k], rph, abort, ea.fault)))) break;
+            if (!(ok = __all_sync(0xffffffffu, mbar_wait(&rbar[k & 1], parity(k), abort, ea.fault)))) break;
+            consumed = k + 1;
             // this thread's row: 16-byte chunk j of the row sits at slot j ^ (row % 8)
-            float4* rowp = reinterpret_cast<float4*>(rbuf + k * C::kResTileBytes + lane * 128);
+            float4* rowp = reinterpret_cast<float4*>(rbuf + (k & 1) * C::kResTileBytes + lane * 128);
             const uint4* bias4 =
                 reinterpret_cast<const uint4*>(static_cast<const bf16*>(ea.bias) + nt * BN + c);
 #pragma unroll
@@ -461,17 +482,25 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0 && row0 < M) {
-              tma_store_2d(&tmR, rbuf + k * C::kResTileBytes, nt * BN + c, row0);
-              bulk_commit_group();
+            if (lane == 0) {
+              if (row0 < M) {
+                tma_store_2d(&tmR, rbuf + (k & 1) * C::kResTileBytes, nt * BN + c, row0);
+                bulk_commit_group();
+              }
+              if (k + 2 < kChunks) {
+                bulk_wait_read_all();    // this chunk's store has read the buffer
+                request(k + 2);
+              }
             }
+            if (k + 2 < kChunks) requested = k + 3;
           }
         }
         if (!ok) {
-          // an aborted pipeline: the residual loads issued above still land first
+          // an aborted pipeline: the residual loads requested above still land first
           int no_abort = 0;
           if (lane == 0)
-            for (int k = 0; k < 2; ++k) mbar_wait(&rbar[k], rph, &no_abort, ea.fault);
+            for (int k = consumed; k < requested; ++k)
+              mbar_wait(&rbar[k & 1], parity(k), &no_abort, ea.fault);
           __syncwarp();
           break;
         }
@@ -505,7 +534,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
     if (lane == 0) abort_peer();
     if constexpr (C::kTmaRes || C::kTmaOut) {
-      if (lane == 0) bulk_wait_all();     // the TMA stores complete before the CTA exits
+      // the TMA stores have read shared memory before the CTA exits; their
+      // writes are complete when the grid is
+      if (lane == 0) bulk_wait_read_all();
     }
   }
   tc_fence_before();
@@ -630,9 +661,7 @@ cudaError_t launch_epi(Epi epi, const void* A, const void* W, int M, int N, int 
     case Epi::BiasGelu: return launch_bn<BN, Epi::BiasGelu, kPair>(A, W, M, N, K, ea, s);
     case Epi::BiasResidualScatter:
       return launch_bn<BN, Epi::BiasResidualScatter, kPair>(A, W, M, N, K, ea, s);
-    case Epi::BiasResidual:
-      // BN = 128 is the TMA residual epilogue, chosen in launch_gemm_tc
-      if constexpr (BN != 128) return launch_bn<BN, Epi::BiasResidual, kPair>(A, W, M, N, K, ea, s);
+    case Epi::BiasResidual:   // chosen in launch_gemm_tc
       break;
   }
   return cudaErrorInvalidValue;
@@ -645,13 +674,10 @@ cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* W, int M, int N, 
   if (M < 1 || K % BK != 0 || N % 64 != 0) return cudaErrorInvalidValue;
   // tiles 128 or 256 columns wide run on CTA pairs (256-row tiles); 64-wide on single CTAs
   if (epi == Epi::BiasResidual) {
-    // a short mainloop (K <= 2048) cannot hide the fp32 residual traffic behind
-    // the MMAs: 128-column tiles with the TMA residual epilogue; a long one keeps
-    // 256-column tiles and the register epilogue
-    if (N % 128 == 0 && (K <= 2048 || N % 256 != 0))
-      return launch_bn<128, Epi::BiasResidual, true>(A, W, M, N, K, ea, s);
-    if (N % 256 == 0) return launch_epi<256, true>(epi, A, W, M, N, K, ea, s);
-    return launch_epi<64, false>(epi, A, W, M, N, K, ea, s);
+    // pair tiles update the fp32 residual stream through the TMA epilogue
+    if (N % 256 == 0) return launch_bn<256, Epi::BiasResidual, true>(A, W, M, N, K, ea, s);
+    if (N % 128 == 0) return launch_bn<128, Epi::BiasResidual, true>(A, W, M, N, K, ea, s);
+    return launch_bn<64, Epi::BiasResidual, false>(A, W, M, N, K, ea, s);
   }
   if (N % 256 == 0) return launch_epi<256, true>(epi, A, W, M, N, K, ea, s);
   if (N % 128 == 0) return launch_epi<128, true>(epi, A, W, M, N, K, ea, s);
