@@ -55,7 +55,12 @@ typedef enum { SR_F32 = 0, SR_BF16 = 1 } sr_dtype;
  *  SR_SEL_TOPK_L2: the K tokens with the largest L2 norm of the last
  *                  dense-early block's output (the activation-norm selector of
  *                  App. B.2, Table 11); ties go to the lower token index.  The
- *                  squared norm is accumulated in fp32. */
+ *                  squared norm of the stored activations (each value rounded
+ *                  to the storage dtype) is accumulated in fp32.  In
+ *                  sr_forward with bf16 storage, n1 >= 1 and D % 128 == 0 the
+ *                  norms come out of the last dense-early block's FC2
+ *                  epilogue; otherwise (and always in sr_select) a separate
+ *                  pass reads the stream. */
 typedef enum { SR_SEL_RANDOM = 0, SR_SEL_TOPK_L2 = 1 } sr_selector;
 
 typedef struct {
@@ -183,7 +188,7 @@ sr_status sr_forward_host(sr_handle* h, const void* x_host, const sr_block_weigh
  * being captured into a CUDA graph. */
 typedef enum {
   SR_KERN_COPY = 0,          /* x -> out device copy when out != x */
-  SR_KERN_SELECT = 1,        /* token selection (and the norms of the top-K selector) */
+  SR_KERN_SELECT = 1,        /* token selection (and the top-K norms when not fused into FC2) */
   SR_KERN_GATHER = 2,        /* h0 = x[:, I, :] (Eq. 8), fused with LN1 of the first
                                 sparse block: reads the selected rows, writes h0 and LN1 */
   SR_KERN_LAYERNORM = 3,

@@ -199,14 +199,16 @@ cudaError_t attention(const sr_handle* h, const void* qkv, void* out, int B, int
 }
 
 // One pre-LN block (Sec. 3.3 Eq. 11) on the fp32 residual stream x [B*T, D], in
-// place.  With `scatter` set this is the last sparse block: its FC2 epilogue
+// place.  With `sqnorm` set, the FC2 epilogue also adds each row's squared norm
+// (values rounded to the storage dtype) to sqnorm [B*T], the scores of the top-K
+// selector.  With `scatter` set this is the last sparse block: its FC2 epilogue
 // writes x0 + (h_out - h0) into the rows idx of the stream `scatter_out`
 // [B*Lx, D] instead of x.  With `gather_from` set this is the first sparse
 // block: its LN1 reads the rows idx of the stream `gather_from` [B*Lx, D]
 // directly and also writes them to x (the gather of Eq. 8, fused).
 sr_status run_block(const sr_handle* hd, float* x, int B, int T, const sr_block_weights& w,
                     bool scatter, float* scatter_out, const int32_t* idx, int Lx,
-                    cudaStream_t s, const float* gather_from = nullptr) {
+                    cudaStream_t s, const float* gather_from = nullptr, float* sqnorm = nullptr) {
   const sr_config& c = hd->cfg;
   const int rows = B * T, D = c.D, H = c.mlp_hidden;
   const double es = double(hd->es), R = double(rows);
@@ -252,7 +254,7 @@ sr_status run_block(const sr_handle* hd, float* x, int B, int T, const sr_block_
   }
   if (!scatter) {
     TraceScope t(hd, SR_KERN_GEMM_FC2, 2.0 * R * D * H, (R * H + 1.0 * D * H + D) * es + 8.0 * R * D, s);
-    sr::EpiArgs e4{w.b2, x, x, nullptr, 0, 0, hd->fault()};
+    sr::EpiArgs e4{w.b2, x, x, nullptr, 0, 0, hd->fault(), sqnorm};
     SR_CUDA(gemm(hd, Epi::BiasResidual, u, w.w2, rows, D, H, e4, s), "fc2 gemm");
   } else {
     // reads h and x0 rows, writes the scattered rows, plus the index set
@@ -272,17 +274,29 @@ bool weights_ok(const sr_block_weights& w) {
   return true;
 }
 
-sr_status do_select(sr_handle* h, const float* x, int32_t K, uint64_t seed, int32_t* idx,
-                    cudaStream_t s) {
+// Whether sr_forward takes the top-K scores from the last dense-early block's FC2
+// epilogue instead of a pass over the stream (the GEMM must be a tcgen05 pair
+// GEMM with the TMA residual epilogue).
+bool scores_fused(const sr_handle* h) {
   const sr_config& c = h->cfg;
+  return c.selector == SR_SEL_TOPK_L2 && h->dt == DType::BF16 && c.n1 > 0 &&
+         sr::gemm_tc_takes_sqnorm(c.D);
+}
+
+// score_ready: the top-K scores are already in the workspace (fused into FC2)
+sr_status do_select(sr_handle* h, const float* x, int32_t K, uint64_t seed, int32_t* idx,
+                    cudaStream_t s, bool score_ready = false) {
+  const sr_config& c = h->cfg;
+  const bool norms = c.selector == SR_SEL_TOPK_L2 && !score_ready;
   const double sel_bytes = 4.0 * c.B * K +
-      (c.selector == SR_SEL_TOPK_L2 ? double(c.B) * c.L * c.D * h->es : 0.0);
+      (c.selector == SR_SEL_TOPK_L2 ? 4.0 * c.B * c.L : 0.0) +
+      (norms ? double(c.B) * c.L * c.D * 4.0 : 0.0);
   TraceScope t(h, SR_KERN_SELECT, 0.0, sel_bytes, s);
   if (c.selector == SR_SEL_RANDOM) {
     SR_CUDA(sr::launch_select_random(c.B, c.L, K, seed, c.shared_indices, idx, s), "select_random");
   } else {
     float* score = static_cast<float*>(h->at(h->plan.score));
-    SR_CUDA(sr::launch_token_sq_norms(h->dt, x, c.B * c.L, c.D, score, s), "token norms");
+    if (norms) SR_CUDA(sr::launch_token_sq_norms(h->dt, x, c.B * c.L, c.D, score, s), "token norms");
     SR_CUDA(sr::launch_select_topk(c.B, c.L, K, score, idx, s), "select_topk");
   }
   return SR_OK;
@@ -394,17 +408,21 @@ sr_status widen_and_early(sr_handle* h, const void* x, const sr_block_weights* w
     h->fault_cleared = true;
   }
   const size_t n = size_t(c.B) * c.L * c.D;
+  // the top-K scores accumulate in the last dense-early block's FC2 epilogue
+  float* score = scores_fused(h) ? static_cast<float*>(h->at(h->plan.score)) : nullptr;
   {
     // the residual stream is held in fp32 for the whole forward
     TraceScope t(h, SR_KERN_COPY, 0.0, double(n) * (h->es + 4.0), s);
-    SR_CUDA(sr::launch_widen(h->dt, x, xs, n, s), "widen x");
+    SR_CUDA(sr::launch_widen(h->dt, x, xs, n, s, score, c.B * c.L), "widen x");
   }
   // every later kernel may start while its predecessor finishes (not while
   // tracing, which records events between kernels)
   const sr::PdlScope pdl(!h->trace);
   sr_status st;
   for (int i = 0; i < c.n1; ++i)
-    if ((st = run_block(h, xs, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
+    if ((st = run_block(h, xs, c.B, c.L, w[i], false, nullptr, nullptr, 0, s, nullptr,
+                        i == c.n1 - 1 ? score : nullptr)) != SR_OK)
+      return st;
   return SR_OK;
 }
 
@@ -419,7 +437,7 @@ sr_status route_and_late(sr_handle* h, float* xs, const sr_block_weights* w, flo
   sr_status st;
   int32_t* idx = idx_out ? idx_out : static_cast<int32_t*>(h->at(h->plan.idx));
   if (route || idx_out)
-    if ((st = do_select(h, xs, K, seed, idx, s)) != SR_OK) return st;
+    if ((st = do_select(h, xs, K, seed, idx, s, scores_fused(h))) != SR_OK) return st;
   if (route) {
     // the gather of Eq. 8 is fused into the first sparse block's LN1
     float* hs = static_cast<float*>(h->at(h->plan.hs));

@@ -449,6 +449,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             for (int k = 2; k < kChunks; ++k) tma_prefetch_l2_2d(&tmR, nt * BN + c_begin + 32 * k, row0);
         }
         int consumed = 0, requested = 2;
+        float sq = 0.f;                  // this thread's row: squares of the bf16-rounded update
         bool ok = __all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault));
         if (ok) {
           tc_fence_after();
@@ -478,6 +479,14 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                 v.z += __uint_as_float(r[4 * j + 2]) + bf16_lo(bw[2 * h2 + 1]);
                 v.w += __uint_as_float(r[4 * j + 3]) + bf16_hi(bw[2 * h2 + 1]);
                 rowp[j ^ (lane & 7)] = v;
+                if (ea.sqnorm) {
+                  const float q4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) {
+                    const float rq = __bfloat162float(__float2bfloat16_rn(q4[e]));
+                    sq = fmaf(rq, rq, sq);
+                  }
+                }
               }
             }
             fence_proxy_async_smem();
@@ -495,6 +504,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if (k + 2 < kChunks) requested = k + 3;
           }
         }
+        // one partial sum per row and tile (the tile's columns of this warp's half)
+        if (ok && ea.sqnorm && row0 + lane < M) atomicAdd(ea.sqnorm + row0 + lane, sq);
         if (!ok) {
           // an aborted pipeline: the residual loads requested above still land first
           int no_abort = 0;
@@ -669,9 +680,12 @@ cudaError_t launch_epi(Epi epi, const void* A, const void* W, int M, int N, int 
 
 }  // namespace
 
+bool gemm_tc_takes_sqnorm(int N) { return N % 128 == 0; }
+
 cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* W, int M, int N, int K,
                            const EpiArgs& ea, cudaStream_t s) {
   if (M < 1 || K % BK != 0 || N % 64 != 0) return cudaErrorInvalidValue;
+  if (ea.sqnorm && (epi != Epi::BiasResidual || !gemm_tc_takes_sqnorm(N))) return cudaErrorInvalidValue;
   // tiles 128 or 256 columns wide run on CTA pairs (256-row tiles); 64-wide on single CTAs
   if (epi == Epi::BiasResidual) {
     // pair tiles update the fp32 residual stream through the TMA epilogue

@@ -67,7 +67,9 @@ cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t*
 int select_max_L();
 
 // ---- storage dtype <-> fp32 residual stream, n elements (n % 8 == 0) ------
-cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream_t s);
+// also zeroes zero[0, nzero) when given
+cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream_t s,
+                         float* zero = nullptr, int nzero = 0);
 // narrow rounds scale * x once to the storage dtype
 cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStream_t s,
                           float scale = 1.0f);
@@ -103,6 +105,8 @@ struct EpiArgs {
   int Kr;               // routed rows per sample (scatter)
   int Lx;               // tokens per sample of the scatter target
   unsigned int* fault;  // fault word (bit 0: a bounded barrier wait timed out)
+  float* sqnorm;        // [M] optional (BiasResidual on pair tiles): += the squares of the
+                        // updated row, each value rounded to bf16 first
 };
 // CUDA-core GEMM (fp32 storage) and tcgen05 GEMM (bf16 storage; K % 64 == 0,
 // N % 64 == 0).
@@ -110,6 +114,8 @@ cudaError_t launch_gemm_simt(DType dt, Epi epi, const void* A, const void* Bw, i
                              int K, const EpiArgs& ea, cudaStream_t s);
 cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* Bw, int M, int N, int K,
                            const EpiArgs& ea, cudaStream_t s);
+// whether launch_gemm_tc takes EpiArgs::sqnorm for a BiasResidual GEMM N columns wide
+bool gemm_tc_takes_sqnorm(int N);
 
 
 // ---- attention core: per (sample, head) softmax(q k^T / sqrt(64)) v ------

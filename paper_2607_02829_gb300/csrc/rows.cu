@@ -86,9 +86,11 @@ layernorm_kernel(const float* __restrict__ x, const T* __restrict__ g, const T* 
 // Storage dtype <-> fp32 stream, n elements (n % 8 == 0), 16-byte vectors.
 template <typename T>
 __global__ void __launch_bounds__(256)
-widen_kernel(const T* __restrict__ x, float* __restrict__ y, size_t nvec) {
+widen_kernel(const T* __restrict__ x, float* __restrict__ y, size_t nvec, float* zero, int nzero) {
   pdl_wait();      // the previous kernel's writes are visible from here
   pdl_trigger();
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nzero; i += gridDim.x * blockDim.x)
+    zero[i] = 0.f;
   constexpr int V = Elem<T>::kVec;
   for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
        i += size_t(gridDim.x) * blockDim.x) {
@@ -156,15 +158,17 @@ template <typename T> int lanes_nv(int D) { return (D / Elem<T>::kVec + 31) / 32
 
 }  // namespace
 
-cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream_t s) {
+cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream_t s,
+                         float* zero, int nzero) {
+  if (!zero) nzero = 0;
   if (dt == DType::BF16) {
     const size_t nvec = n / 8;
     return launch_k(widen_kernel<bf16>, dim3(grid_for(nvec)), dim3(256), 0, s, 1,
-                    static_cast<const bf16*>(x), y, nvec);
+                    static_cast<const bf16*>(x), y, nvec, zero, nzero);
   }
   const size_t nvec = n / 4;
   return launch_k(widen_kernel<float>, dim3(grid_for(nvec)), dim3(256), 0, s, 1,
-                  static_cast<const float*>(x), y, nvec);
+                  static_cast<const float*>(x), y, nvec, zero, nzero);
 }
 
 cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStream_t s, float scale) {

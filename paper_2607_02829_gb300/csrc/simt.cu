@@ -180,6 +180,7 @@ cudaError_t gemm_simt_t(Epi epi, const void* A, const void* Bw, int M, int N, in
 
 cudaError_t launch_gemm_simt(DType dt, Epi epi, const void* A, const void* Bw, int M, int N,
                              int K, const EpiArgs& ea, cudaStream_t s) {
+  if (ea.sqnorm) return cudaErrorInvalidValue;     // row norms are fused on the tcgen05 path only
   if (dt == DType::F32) return gemm_simt_t<float>(epi, A, Bw, M, N, K, ea, s);
   return gemm_simt_t<bf16>(epi, A, Bw, M, N, K, ea, s);
 }

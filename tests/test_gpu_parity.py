@@ -162,14 +162,17 @@ def test_forward_parity_workload(wlname):
     assert err <= TOL[wl.dtype], err
 
 
-def test_forward_parity_topk_selector_small():
-    wl = _tiny("bf16", B=2, L=256, heads=2, split=(1, 2, 1), r=0.25, selector="topk_l2")
+# bf16 with D = 128: the scores come from the dense-early block's FC2 epilogue;
+# D = 192 (64-column GEMM tiles) and fp32 take the separate pass over the stream
+@pytest.mark.parametrize("dtype,heads", [("bf16", 2), ("bf16", 3), ("f32", 2)])
+def test_forward_parity_topk_selector_small(dtype, heads):
+    wl = _tiny(dtype, B=2, L=256, heads=heads, split=(2, 2, 1), r=0.25, selector="topk_l2")
     x, ws = synth.make_inputs(wl)
     out, idx = gpu_forward(wl, x, ws)
     ref, ridx = _oracle(wl, x, ws, idx=idx)      # same indices on both sides
     err = max_norm_rel(synth.stored_as_f64(out), ref)
-    assert err <= TOL["bf16"], err
-    x0, _ = gpu_forward(wl, x, ws, n_split=(1, 0, 0), want_idx=False)
+    assert err <= TOL[dtype], err
+    x0, _ = gpu_forward(wl, x, ws, n_split=(2, 0, 0), want_idx=False)
     assert np.array_equal(idx, o.select_topk_l2(synth.stored_as_f64(x0), 64))
 
 
