@@ -18,6 +18,7 @@ import json
 import os
 import subprocess
 import sys
+import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -77,15 +78,19 @@ class ClockSampler:
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index):
+    def __init__(self, gpu_index, keep_path=None):
         self.gpu = gpu_index
         self.proc = None
         self.path = None
+        self.keep_path = keep_path       # raw samples are kept only when asked for
 
     def start(self):
         try:
-            os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
-            self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+            if self.keep_path:
+                self.path = self.keep_path
+            else:
+                fd, self.path = tempfile.mkstemp(prefix="sr_clocks_", suffix=".csv")
+                os.close(fd)
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
@@ -118,6 +123,11 @@ class ClockSampler:
                 for n, v in zip(names, p[5:9]):
                     if v.lower() == "active":
                         reasons.add(n)
+        if not self.keep_path:
+            try:
+                os.remove(self.path)
+            except OSError:
+                pass
         if not sm:
             return None
         sm.sort()
@@ -189,7 +199,7 @@ def run_ours(args, rank, world, local_rank):
     # ---- timed region: K steps, L2 flushed before each, events around each step
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
-    clocks = ClockSampler(local_rank)
+    clocks = ClockSampler(local_rank, args.clocks_csv)
     clocks.start()
     barrier()
     torch.cuda.synchronize()
@@ -353,6 +363,8 @@ def main():
                     help="override the block split n1,n2,n3 (kernel studies and profiling)")
     ap.add_argument("--sweep", choices=["gather", "ensemble", "cross_attention"], default=None,
                     help="size sweep of one kernel (prints one JSON line per size)")
+    ap.add_argument("--clocks-csv", default=None,
+                    help="keep the raw nvidia-smi samples of the timed region in this file")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
