@@ -2,6 +2,7 @@
 // the launch sequence of Alg. 1 (dense early -> select -> gather -> sparse
 // middle -> delta scatter -> dense late).  Everything here is host code; every
 // step of the computation runs in the kernels it launches.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -90,7 +91,9 @@ Plan make_plan(const sr_config& c, int32_t Kmax) {
   p.u = off;     off += align_up(brows * size_t(c.mlp_hidden) * es);
   p.hs = off;    off += align_up(rrows * c.D * sizeof(float));    // fp32 routed stream
   p.idx = off;   off += align_up(size_t(c.B) * c.L * sizeof(int32_t));
-  p.score = off; off += align_up(rows * sizeof(float));
+  // top-K scores: one per token, or the FC2 epilogue's partial sums per token
+  const int parts = c.dtype == SR_BF16 ? std::max(1, sr::gemm_tc_sqnorm_parts(c.D)) : 1;
+  p.score = off; off += align_up(rows * size_t(parts) * sizeof(float));
   p.total = off;
   return p;
 }
@@ -199,9 +202,9 @@ cudaError_t attention(const sr_handle* h, const void* qkv, void* out, int B, int
 }
 
 // One pre-LN block (Sec. 3.3 Eq. 11) on the fp32 residual stream x [B*T, D], in
-// place.  With `sqnorm` set, the FC2 epilogue also adds each row's squared norm
-// (values rounded to the storage dtype) to sqnorm [B*T], the scores of the top-K
-// selector.  With `scatter` set this is the last sparse block: its FC2 epilogue
+// place.  With `sqnorm` set, the FC2 epilogue also writes each row's squared
+// norm (values rounded to the storage dtype) as partial sums per half tile to
+// sqnorm [B*T][parts], the scores of the top-K selector.  With `scatter` set this is the last sparse block: its FC2 epilogue
 // writes x0 + (h_out - h0) into the rows idx of the stream `scatter_out`
 // [B*Lx, D] instead of x.  With `gather_from` set this is the first sparse
 // block: its LN1 reads the rows idx of the stream `gather_from` [B*Lx, D]
@@ -280,7 +283,7 @@ bool weights_ok(const sr_block_weights& w) {
 bool scores_fused(const sr_handle* h) {
   const sr_config& c = h->cfg;
   return c.selector == SR_SEL_TOPK_L2 && h->dt == DType::BF16 && c.n1 > 0 &&
-         sr::gemm_tc_takes_sqnorm(c.D);
+         sr::gemm_tc_sqnorm_parts(c.D) > 0;
 }
 
 // score_ready: the top-K scores are already in the workspace (fused into FC2)
@@ -297,7 +300,8 @@ sr_status do_select(sr_handle* h, const float* x, int32_t K, uint64_t seed, int3
   } else {
     float* score = static_cast<float*>(h->at(h->plan.score));
     if (norms) SR_CUDA(sr::launch_token_sq_norms(h->dt, x, c.B * c.L, c.D, score, s), "token norms");
-    SR_CUDA(sr::launch_select_topk(c.B, c.L, K, score, idx, s), "select_topk");
+    const int parts = norms ? 1 : sr::gemm_tc_sqnorm_parts(c.D);
+    SR_CUDA(sr::launch_select_topk(c.B, c.L, K, score, idx, s, parts), "select_topk");
   }
   return SR_OK;
 }
@@ -408,12 +412,13 @@ sr_status widen_and_early(sr_handle* h, const void* x, const sr_block_weights* w
     h->fault_cleared = true;
   }
   const size_t n = size_t(c.B) * c.L * c.D;
-  // the top-K scores accumulate in the last dense-early block's FC2 epilogue
+  // the top-K scores come out of the last dense-early block's FC2 epilogue as
+  // partial sums per row
   float* score = scores_fused(h) ? static_cast<float*>(h->at(h->plan.score)) : nullptr;
   {
     // the residual stream is held in fp32 for the whole forward
     TraceScope t(h, SR_KERN_COPY, 0.0, double(n) * (h->es + 4.0), s);
-    SR_CUDA(sr::launch_widen(h->dt, x, xs, n, s, score, c.B * c.L), "widen x");
+    SR_CUDA(sr::launch_widen(h->dt, x, xs, n, s), "widen x");
   }
   // every later kernel may start while its predecessor finishes (not while
   // tracing, which records events between kernels)

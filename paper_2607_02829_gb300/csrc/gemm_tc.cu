@@ -504,8 +504,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if (k + 2 < kChunks) requested = k + 3;
           }
         }
-        // one partial sum per row and tile (the tile's columns of this warp's half)
-        if (ok && ea.sqnorm && row0 + lane < M) atomicAdd(ea.sqnorm + row0 + lane, sq);
+        // one partial sum per row and half tile, in its own slot (the sum over the
+        // slots is taken in a fixed order, so the scores are reproducible)
+        if (ok && ea.sqnorm && row0 + lane < M)
+          ea.sqnorm[size_t(row0 + lane) * (2 * n_tiles) + (nt * 2 + half)] = sq;
         if (!ok) {
           // an aborted pipeline: the residual loads requested above still land first
           int no_abort = 0;
@@ -680,12 +682,17 @@ cudaError_t launch_epi(Epi epi, const void* A, const void* W, int M, int N, int 
 
 }  // namespace
 
-bool gemm_tc_takes_sqnorm(int N) { return N % 128 == 0; }
+int gemm_tc_sqnorm_parts(int N) {
+  // BiasResidual runs 256-column pair tiles when 256 divides N, else 128-column ones
+  if (N % 256 == 0) return N / 128;
+  if (N % 128 == 0) return N / 64;
+  return 0;
+}
 
 cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* W, int M, int N, int K,
                            const EpiArgs& ea, cudaStream_t s) {
   if (M < 1 || K % BK != 0 || N % 64 != 0) return cudaErrorInvalidValue;
-  if (ea.sqnorm && (epi != Epi::BiasResidual || !gemm_tc_takes_sqnorm(N))) return cudaErrorInvalidValue;
+  if (ea.sqnorm && (epi != Epi::BiasResidual || gemm_tc_sqnorm_parts(N) == 0)) return cudaErrorInvalidValue;
   // tiles 128 or 256 columns wide run on CTA pairs (256-row tiles); 64-wide on single CTAs
   if (epi == Epi::BiasResidual) {
     // pair tiles update the fp32 residual stream through the TMA epilogue

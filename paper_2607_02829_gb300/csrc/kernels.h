@@ -60,9 +60,11 @@ cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared,
 // stores), its square accumulated in fp32.
 cudaError_t launch_token_sq_norms(DType dt, const float* x, int rows, int D, float* score,
                                   cudaStream_t s);
-// K largest scores per sample (ties to the lower index), sorted indices.
+// K largest scores per sample (ties to the lower index), sorted indices.  A
+// token's score is the sum of `parts` consecutive partial sums (score
+// [B*L][parts]), added in order.
 cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t* idx,
-                               cudaStream_t s);
+                               cudaStream_t s, int parts = 1);
 // Largest L the one-CTA-per-sample selection kernels accept (keys in shared memory).
 int select_max_L();
 
@@ -105,8 +107,9 @@ struct EpiArgs {
   int Kr;               // routed rows per sample (scatter)
   int Lx;               // tokens per sample of the scatter target
   unsigned int* fault;  // fault word (bit 0: a bounded barrier wait timed out)
-  float* sqnorm;        // [M] optional (BiasResidual on pair tiles): += the squares of the
-                        // updated row, each value rounded to bf16 first
+  float* sqnorm;        // [M][2N/BN] optional (BiasResidual on pair tiles): per row, one sum
+                        // of squares of the updated values (each rounded to bf16 first)
+                        // for each half tile of BN/2 columns, in column order
 };
 // CUDA-core GEMM (fp32 storage) and tcgen05 GEMM (bf16 storage; K % 64 == 0,
 // N % 64 == 0).
@@ -114,8 +117,9 @@ cudaError_t launch_gemm_simt(DType dt, Epi epi, const void* A, const void* Bw, i
                              int K, const EpiArgs& ea, cudaStream_t s);
 cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* Bw, int M, int N, int K,
                            const EpiArgs& ea, cudaStream_t s);
-// whether launch_gemm_tc takes EpiArgs::sqnorm for a BiasResidual GEMM N columns wide
-bool gemm_tc_takes_sqnorm(int N);
+// partial sums per row that launch_gemm_tc writes to EpiArgs::sqnorm for a
+// BiasResidual GEMM N columns wide; 0 when it does not take sqnorm
+int gemm_tc_sqnorm_parts(int N);
 
 
 // ---- attention core: per (sample, head) softmax(q k^T / sqrt(64)) v ------

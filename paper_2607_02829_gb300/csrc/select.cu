@@ -147,14 +147,20 @@ select_random_kernel(int L, int K, uint64_t seed, int shared, int32_t* idx) {
 }
 
 __global__ void __launch_bounds__(kSelThreads)
-select_topk_kernel(int L, int K, const float* __restrict__ score, int32_t* idx) {
+select_topk_kernel(int L, int K, const float* __restrict__ score, int parts, int32_t* idx) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   pdl_wait();      // the previous kernel's writes are visible from here
   pdl_trigger();
 
   uint32_t* keys = reinterpret_cast<uint32_t*>(smem_raw);
   const int b = blockIdx.x;
-  for (int i = threadIdx.x; i < L; i += blockDim.x) keys[i] = desc_key(score[size_t(b) * L + i]);
+  // a token's score is the sum of its `parts` partial sums, added in slot order
+  for (int i = threadIdx.x; i < L; i += blockDim.x) {
+    const float* sp = score + (size_t(b) * L + i) * parts;
+    float v = sp[0];
+    for (int p = 1; p < parts; ++p) v += sp[p];
+    keys[i] = desc_key(v);
+  }
   __syncthreads();
   select_smallest_sorted<uint32_t>(keys, L, K, idx + size_t(b) * K);
 }
@@ -200,12 +206,12 @@ cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared,
 }
 
 cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t* idx,
-                               cudaStream_t s) {
+                               cudaStream_t s, int parts) {
   const size_t smem = size_t(L) * sizeof(uint32_t);
   cudaError_t e = cudaFuncSetAttribute(select_topk_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
-  return launch_k(select_topk_kernel, dim3(B), dim3(kSelThreads), smem, s, 1, L, K, score, idx);
+  return launch_k(select_topk_kernel, dim3(B), dim3(kSelThreads), smem, s, 1, L, K, score, parts, idx);
 }
 
 cudaError_t launch_token_sq_norms(DType dt, const float* x, int rows, int D, float* score,

@@ -174,6 +174,8 @@ def test_forward_parity_topk_selector_small(dtype, heads):
     assert err <= TOL[dtype], err
     x0, _ = gpu_forward(wl, x, ws, n_split=(2, 0, 0), want_idx=False)
     assert np.array_equal(idx, o.select_topk_l2(synth.stored_as_f64(x0), 64))
+    again, idx2 = gpu_forward(wl, x, ws)
+    assert torch.equal(out, again) and np.array_equal(idx, idx2)     # reproducible
 
 
 # ------------------------------------------------------------ implicit ensemble
