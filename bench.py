@@ -254,23 +254,50 @@ def run_ours(args, rank, world, local_rank):
                    "tflops": seg_flops / (seg_ms * 1e-3) / 1e12}
         senc.close()
 
-    # ---- end to end through the C ABI from pinned host memory
+    # ---- end to end through the C ABI from pinned host memory.  Every step copies
+    # its input in and its result out; the copies run on their own streams, so
+    # step i + 1's input and step i - 1's result move while step i computes
+    # (two device and two pinned host buffers, ordered by events).
     xh = x_cpu.pin_memory()
-    oh = torch.empty_like(xh).pin_memory()
-    dbuf = torch.empty_like(x)
+    oh = [torch.empty_like(xh).pin_memory() for _ in range(2)]
+    din = [torch.empty_like(x) for _ in range(2)]
+    dout = [torch.empty_like(x) for _ in range(2)]
     bytes_io = x.numel() * x.element_size()
-    for i in range(max(1, args.warmup // 2)):
-        b.sr_forward_host(enc.handle, xh.data_ptr(), warr, wl.keep_ratio, seed, dbuf.data_ptr(),
-                          oh.data_ptr(), None, stream.cuda_stream)
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    fwd_done = [torch.cuda.Event() for _ in range(2)]
+    in_ready = [torch.cuda.Event() for _ in range(2)]
+    out_read = [torch.cuda.Event() for _ in range(2)]
+
+    def e2e_step(i):
+        k = i % 2
+        if i >= 2:
+            s_in.wait_event(fwd_done[k])        # forward i - 2 has read din[k]
+        with torch.cuda.stream(s_in):
+            din[k].copy_(xh, non_blocking=True)
+        in_ready[k].record(s_in)
+        stream.wait_event(in_ready[k])
+        if i >= 2:
+            stream.wait_event(out_read[k])      # step i - 2's result has left dout[k]
+        b.sr_forward(enc.handle, din[k].data_ptr(), warr, wl.keep_ratio, seed + i,
+                     dout[k].data_ptr(), None, stream.cuda_stream)
+        fwd_done[k].record(stream)
+        s_out.wait_event(fwd_done[k])
+        with torch.cuda.stream(s_out):
+            oh[k].copy_(dout[k], non_blocking=True)
+        out_read[k].record(s_out)
+
+    for i in range(max(2, args.warmup // 2)):
+        e2e_step(i)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
-    e0.record(stream)
+    e0.record(s_in)
     for i in range(args.steps):
-        b.sr_forward_host(enc.handle, xh.data_ptr(), warr, wl.keep_ratio, seed + i,
-                          dbuf.data_ptr(), oh.data_ptr(), None, stream.cuda_stream)
-    e1.record(stream)
+        e2e_step(i)
+    e1.record(s_out)
     torch.cuda.synchronize()
+    if not torch.equal(oh[(args.steps - 1) % 2], dout[(args.steps - 1) % 2].cpu()):
+        raise RuntimeError("end-to-end result differs from the device result")
     e2e_ms = e0.elapsed_time(e1) / args.steps
     e2e_ms = max_over_ranks(e2e_ms, world, dev)
     enc.close()

@@ -151,6 +151,30 @@ def test_forward_parity_small(dtype, B, L, heads, split, r):
     assert err <= TOL[dtype], err
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_forward_host_equals_device_forward(dtype):
+    # the one-call host form: copy in, sr_forward in place, copy out
+    from paper_2607_02829_gb300 import binding as b
+    wl = _tiny(dtype, B=2, L=200, heads=2, split=(1, 2, 1), r=0.25)
+    x, ws = synth.make_inputs(wl)
+    ref, ridx = gpu_forward(wl, x, ws)
+    cfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, wl.n1, wl.n2, wl.n3, dtype=dtype)
+    enc = b.Encoder(cfg, max_keep_ratio=wl.keep_ratio)
+    wd = [{k: v.cuda() for k, v in blk.items()} for blk in ws[:wl.N]]
+    warr = b.weights_array(wd)
+    xh = x.pin_memory()
+    oh = torch.empty_like(xh).pin_memory()
+    dbuf = torch.empty_like(x, device="cuda")
+    idx = torch.empty(wl.B, 50, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream()
+    b.sr_forward_host(enc.handle, xh.data_ptr(), warr, wl.keep_ratio, wl.select_seed,
+                      dbuf.data_ptr(), oh.data_ptr(), idx.data_ptr(), stream.cuda_stream)
+    torch.cuda.synchronize()
+    assert torch.equal(oh, ref)
+    assert np.array_equal(idx.cpu().numpy().astype(np.int64), ridx)
+    enc.close()
+
+
 @pytest.mark.parametrize("wlname", ["c1_5p625deg_f32", "c2_5p625deg_bf16"])
 def test_forward_parity_workload(wlname):
     wl = synth.WORKLOADS[wlname]
