@@ -36,9 +36,11 @@ struct GemmCfg {
   // each loads its own 128 rows of A and half of the tile's B rows
   static constexpr int kRowsTile = kPair ? 2 * BM : BM;
   static constexpr int kBRows = kPair ? BN / 2 : BN;
-  // the residual epilogue of pair tiles keeps two 32 x 32 fp32 residual tiles
-  // per epilogue warp in shared memory (64 KB), paid for with a shorter operand
-  // ring on 256-column tiles
+  // the residual epilogue of pair tiles stages two 32 x 32 fp32 chunks per
+  // epilogue warp in shared memory (64 KB), paid for with a shorter operand ring
+  // on 256-column tiles: bias + accumulator, added into the stream by TMA
+  // reduce; or, when the updated rows' norms are wanted, the residual itself,
+  // loaded by TMA, updated in place and stored back
   static constexpr bool kTmaRes = E == Epi::BiasResidual && kPair;
   // bf16 outputs of tiles at least 128 columns wide leave through TMA stores
   // from a 128-byte-swizzled 32 x 64 tile per epilogue warp (4 KB)
@@ -431,6 +433,46 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         unsigned char* rbuf = reinterpret_cast<unsigned char*>(staging) +
                               size_t(warp - 2) * 2 * C::kResTileBytes;
         uint64_t* rbar = sm->res_full[warp - 2];
+        if (!ea.sqnorm) {
+          // bias + accumulator staged per chunk and added into the stream by TMA
+          // reduce: the residual itself never passes through the SM
+          if (!__all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault))) break;
+          tc_fence_after();
+          const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
+#pragma unroll 1
+          for (int k = 0; k < kChunks; ++k) {
+            const int c = c_begin + 32 * k;
+            uint32_t r[32];
+            tmem_ld32(tbase + uint32_t(c), r);
+            tmem_wait_ld();
+            // the buffer's previous reduce (two chunks back) has read it
+            if (lane == 0) bulk_wait_read_le1();
+            __syncwarp();
+            float4* rowp = reinterpret_cast<float4*>(rbuf + (k & 1) * C::kResTileBytes + lane * 128);
+            const uint4* bias4 =
+                reinterpret_cast<const uint4*>(static_cast<const bf16*>(ea.bias) + nt * BN + c);
+#pragma unroll
+            for (int jq = 0; jq < 4; ++jq) {
+              const uint4 bq = __ldg(bias4 + jq);
+              const uint32_t bw[4] = {bq.x, bq.y, bq.z, bq.w};
+#pragma unroll
+              for (int h2 = 0; h2 < 2; ++h2) {
+                const int j = 2 * jq + h2;
+                rowp[j ^ (lane & 7)] =
+                    make_float4(__uint_as_float(r[4 * j]) + bf16_lo(bw[2 * h2]),
+                                __uint_as_float(r[4 * j + 1]) + bf16_hi(bw[2 * h2]),
+                                __uint_as_float(r[4 * j + 2]) + bf16_lo(bw[2 * h2 + 1]),
+                                __uint_as_float(r[4 * j + 3]) + bf16_hi(bw[2 * h2 + 1]));
+              }
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0 && row0 < M) {
+              tma_reduce_add_2d(&tmR, rbuf + (k & 1) * C::kResTileBytes, nt * BN + c, row0);
+              bulk_commit_group();
+            }
+          }
+        } else {
         auto request = [&](int k) {   // lane 0 only
           mbar_arrive_expect_tx(&rbar[k & 1], C::kResTileBytes);
           tma_load_2d(&tmR, rbuf + (k & 1) * C::kResTileBytes, &rbar[k & 1],
@@ -516,6 +558,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               mbar_wait(&rbar[k & 1], parity(k), &no_abort, ea.fault);
           __syncwarp();
           break;
+        }
         }
       } else {
         // the first chunk's residual loads overlap the wait for the accumulator
