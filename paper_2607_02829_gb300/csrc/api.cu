@@ -583,11 +583,17 @@ sr_status sr_forward_host(sr_handle* h, const void* x_host, const sr_block_weigh
   if (!h) return fail(SR_ERR_INVALID_ARG, "handle is NULL");
   if (!x_host || !out_host || !dev_xout)
     return fail(SR_ERR_INVALID_ARG, "x_host, dev_xout and out_host must be non-NULL");
+  // every argument is checked before the first copy is enqueued
+  int32_t K = 0;
+  sr_status st = check_forward_args(h, dev_xout, w, keep_ratio, dev_xout, &K);
+  if (st != SR_OK) return st;
+  if (idx_out && !aligned(idx_out, 4)) return fail(SR_ERR_INVALID_ARG, "idx_out misaligned");
+  if (idx_out && K < 1) return fail(SR_ERR_INVALID_ARG, "K = floor(L * keep_ratio) is 0");
   const sr_config& c = h->cfg;
   const size_t bytes = size_t(c.B) * c.L * c.D * h->es;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   SR_CUDA(cudaMemcpyAsync(dev_xout, x_host, bytes, cudaMemcpyHostToDevice, s), "copy x host -> device");
-  sr_status st = sr_forward(h, dev_xout, w, keep_ratio, seed, dev_xout, idx_out, stream);
+  st = sr_forward(h, dev_xout, w, keep_ratio, seed, dev_xout, idx_out, stream);
   if (st != SR_OK) return st;
   SR_CUDA(cudaMemcpyAsync(out_host, dev_xout, bytes, cudaMemcpyDeviceToHost, s), "copy out device -> host");
   return SR_OK;

@@ -179,3 +179,35 @@ def test_cross_attention_argument_errors(L):
             b.sr_cross_attention(a["q"], a["kv"], a["B"], a["Tq"], a["Tkv"], a["heads"], a["out"],
                                  a["fault"], a["stream"])
         assert e.value.status == status, kw
+
+
+def test_forward_host_rejects_arguments_before_any_copy(L):
+    # every check runs on the host before the first copy is enqueued, so fake
+    # addresses are never touched
+    from paper_2607_02829_gb300 import binding as b
+    cfg = b.make_config(2, 512, 256, 4, 1, 2, 1, dtype="bf16")
+    h = _handle(b, cfg, b.sr_workspace_bytes(cfg, 0.25))
+    try:
+        w = (b.sr_block_weights * 4)()
+        for i in range(4):
+            for f in b.WEIGHT_FIELDS:
+                setattr(w[i], f, 0x200000)
+        XH, D, OH = 0x7000000, 0x400000, 0x8000000
+        for args, status in [
+            ((None, w, 0.25, D, OH), b.SR_ERR_INVALID_ARG),       # no host input
+            ((XH, w, 0.25, None, OH), b.SR_ERR_INVALID_ARG),      # no device buffer
+            ((XH, w, 0.25, D, None), b.SR_ERR_INVALID_ARG),       # no host output
+            ((XH, w, 1.5, D, OH), b.SR_ERR_INVALID_ARG),          # keep ratio out of range
+            ((XH, w, 0.5, D, OH), b.SR_ERR_WORKSPACE),            # beyond the routed capacity
+            ((XH, w, 0.25, D + 8, OH), b.SR_ERR_INVALID_ARG),     # misaligned device buffer
+        ]:
+            x_host, ww, r, dev, out_host = args
+            with pytest.raises(b.SRError) as e:
+                b.sr_forward_host(h, x_host, ww, r, 0, dev, out_host, None, None)
+            assert e.value.status == status, args
+        w[2].w2 = None                                         # a NULL weight pointer
+        with pytest.raises(b.SRError) as e:
+            b.sr_forward_host(h, XH, w, 0.25, 0, D, OH, None, None)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+    finally:
+        b.sr_destroy(h)
