@@ -57,3 +57,45 @@ def test_single_rank_helpers_without_a_process_group():
     import bench
     assert bench.max_over_ranks(3.5, 1, torch.device("cpu")) == 3.5
     assert bench.job_tokens_per_s(1000, 1, 2.0) == pytest.approx(500000.0)
+
+
+def _run_bench(args, env_extra=None, timeout=300):
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ)
+    for k in ("RANK", "WORLD_SIZE", "LOCAL_RANK"):
+        env.pop(k, None)
+    env.update(env_extra or {})
+    r = subprocess.run([sys.executable, os.path.join(root, "bench.py")] + args, cwd=root, env=env,
+                       capture_output=True, text=True, timeout=timeout)
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    return r.returncode, [json.loads(l) for l in lines]
+
+
+def test_reference_arm_prints_the_contract_line():
+    # the reference arm times the oracle on the host cores; on the small fp32
+    # workload it finishes in seconds and needs no GPU
+    rc, lines = _run_bench(["--impl", "reference", "--workload", "c1_5p625deg_f32",
+                            "--steps", "1", "--warmup", "3"])
+    assert rc == 0 and len(lines) == 1
+    d = lines[0]
+    assert d["impl"] == "reference"
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+                "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config",
+                "cpu_baseline", "e2e"):
+        assert key in d, key
+    assert d["value"] > 0 and d["steps"] == 1 and d["warmup"] >= 3 and d["higher_is_better"] is True
+    assert d["config"]["workload"] == "c1_5p625deg_f32"
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}
+
+
+def test_reference_arm_other_ranks_exit_without_work():
+    rc, lines = _run_bench(["--impl", "reference", "--workload", "c1_5p625deg_f32",
+                            "--steps", "1", "--warmup", "3", "--gpus", "2"],
+                           {"RANK": "1", "WORLD_SIZE": "2", "LOCAL_RANK": "1"}, timeout=120)
+    assert rc == 0 and lines == []
