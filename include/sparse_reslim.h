@@ -122,8 +122,12 @@ sr_status sr_select(sr_handle* h, const void* x, float keep_ratio, uint64_t seed
  *            only read during the call.
  *  out     : [B, L, D] device output; may equal x (in place) but must not
  *            otherwise overlap it.
- *  idx_out : optional [B, K] int32 device buffer that receives the index set
- *            (identical to sr_select's for the same arguments), or NULL.
+ *  idx_out : optional [B, K] int32 device buffer that receives the index set,
+ *            or NULL.  With SR_SEL_RANDOM it is identical to sr_select's for
+ *            the same arguments.  SR_SEL_TOPK_L2 ranks the output of the last
+ *            dense-early block (x itself when n1 == 0); sr_select given that
+ *            tensor picks the same set up to ties of the fp32 scores (the
+ *            sums are added in a different order).
  * keep_ratio == 1 runs the plain dense stack (Sec. 3.4, "Architecture-agnostic design": r = 1 is the dense
  * baseline), with no selection, gather or scatter; n2 == 0 likewise routes
  * nothing.  Unselected rows of out are bit-identical to the input of the first

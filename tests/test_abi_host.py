@@ -211,3 +211,19 @@ def test_forward_host_rejects_arguments_before_any_copy(L):
         assert e.value.status == b.SR_ERR_INVALID_ARG
     finally:
         b.sr_destroy(h)
+
+
+@pytest.mark.parametrize("lang", ["c", "c++"])
+def test_header_compiles_as_plain_c_and_cpp(lang):
+    # the boundary is a C header: it must stand alone in a C and a C++ unit
+    import os
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc" if lang == "c" else "g++")
+    if cc is None:
+        pytest.skip("no host compiler")
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([cc, "-fsyntax-only", "-Wall", "-Werror", "-x", lang,
+                        os.path.join(root, "include", "sparse_reslim.h")],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
