@@ -227,3 +227,49 @@ def test_header_compiles_as_plain_c_and_cpp(lang):
                         os.path.join(root, "include", "sparse_reslim.h")],
                        capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
+
+
+def test_trace_fault_and_error_message_arguments(L):
+    from paper_2607_02829_gb300 import binding as b
+    assert L.sr_trace_enable(None, 1) == b.SR_ERR_INVALID_ARG
+    assert L.sr_trace_read(None, None, 0) == b.SR_ERR_INVALID_ARG
+    f = ctypes.c_uint32(7)
+    assert L.sr_device_fault(None, ctypes.byref(f), 0, None) == b.SR_ERR_INVALID_ARG
+    assert b"NULL" in L.sr_last_error_message()          # the message of that rejection
+    cfg = b.make_config(2, 512, 256, 4, 1, 2, 1, dtype="bf16")
+    h = _handle(b, cfg, b.sr_workspace_bytes(cfg, 0.25))
+    try:
+        # nothing traced yet: the read needs no device work and gives zeros
+        assert L.sr_trace_enable(h, 1) == b.SR_OK
+        buf = (b.sr_trace_entry * 10)()
+        assert L.sr_trace_read(h, buf, 1) == b.SR_OK
+        assert all(e.launches == 0 and e.ms == 0.0 and e.flops == 0.0 for e in buf)
+        assert L.sr_trace_enable(h, 0) == b.SR_OK
+        assert L.sr_device_fault(h, None, 0, None) == b.SR_ERR_INVALID_ARG
+    finally:
+        b.sr_destroy(h)
+
+
+def test_static_topk_selector_rejects_arguments_before_any_launch(L):
+    # x, B, L, D, dtype, keep_ratio, idx -> status; fake addresses are never touched
+    from paper_2607_02829_gb300 import binding as b
+    X, I = 0x400000, 0x800000
+    good = dict(x=X, B=2, L=512, D=256, dtype=b.SR_BF16, r=0.25, idx=I)
+    cases = [
+        (dict(x=None), b.SR_ERR_INVALID_ARG), (dict(x=X + 8), b.SR_ERR_INVALID_ARG),
+        (dict(idx=None), b.SR_ERR_INVALID_ARG), (dict(idx=I + 2), b.SR_ERR_INVALID_ARG),
+        (dict(dtype=7), b.SR_ERR_INVALID_ARG), (dict(B=0), b.SR_ERR_INVALID_ARG),
+        (dict(L=0), b.SR_ERR_INVALID_ARG), (dict(D=100), b.SR_ERR_UNSUPPORTED),
+        (dict(D=4096), b.SR_ERR_UNSUPPORTED), (dict(D=2048, dtype=b.SR_F32), b.SR_ERR_UNSUPPORTED),
+        (dict(B=65, L=16200), b.SR_ERR_UNSUPPORTED),        # B * L above the 1,048,576 scores
+        (dict(r=0.0), b.SR_ERR_INVALID_ARG), (dict(r=1.5), b.SR_ERR_INVALID_ARG),
+        (dict(r=float("nan")), b.SR_ERR_INVALID_ARG),
+        (dict(L=10, r=0.05), b.SR_ERR_INVALID_ARG),         # K = floor(0.5) = 0
+    ]
+    for kw, status in cases:
+        a = dict(good, **kw)
+        k = ctypes.c_int32(-1)
+        got = L.sr_select_topk_l2_static(a["x"], a["B"], a["L"], a["D"], a["dtype"], a["r"],
+                                         a["idx"], ctypes.byref(k), None)
+        assert got == status, (kw, got)
+        assert k.value == -1                                # K_out untouched on a rejection
