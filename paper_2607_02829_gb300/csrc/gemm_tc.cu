@@ -2,17 +2,23 @@
 // the block's epilogues fused (bias; bias + GELU; bias + fp32 residual add; bias
 // + residual + the delta scatter of Eq. 9 for the last sparse block).
 //
-// Persistent, warp-specialised, one CTA per SM (320 threads):
-//   warp 0      TMA producer: A and B tiles (128 x 64 and BN x 64 bf16, 128-byte
-//               swizzle) into a ring of shared-memory stages;
-//   warp 1      owns the tensor memory and issues tcgen05.mma (M = 128, N = BN,
-//               K = 16) into one of two TMEM accumulators;
+// Persistent and warp-specialised, 320 threads per CTA.  Tiles 128 or 256
+// columns wide run on CTA pairs (clusters of two, tcgen05.mma.cta_group::2):
+// the pair shares a 256-row tile, each CTA holding 128 rows of A and half of
+// the tile's B rows; 64-column tiles run on single CTAs (M = 128).
+//   warp 0      TMA producer: A and B tiles (64 columns of K, 128-byte swizzle)
+//               into a ring of shared-memory stages; a pair's loads complete on
+//               the even CTA's stage barrier;
+//   warp 1      owns the tensor memory; of a pair only the even CTA issues the
+//               MMAs (K = 16 each), into one of two TMEM accumulators;
 //   warps 2..9  epilogue: tcgen05.ld of the finished accumulator (one row per
 //               thread; two warps per TMEM lane quarter, each taking half of
-//               the tile's columns), the fused epilogue, then a per-warp
-//               shared-memory transpose so that every global load and store
-//               covers whole row segments; the second accumulator lets the
-//               next tile's MMAs run meanwhile.
+//               the tile's columns) while the other accumulator takes the next
+//               tile's MMAs.  bf16 outputs leave through TMA stores of
+//               swizzled shared-memory tiles; the fp32 residual is updated by
+//               TMA reduce (bias + accumulator added into the stream in L2);
+//               the scatter and 64-column tiles use a per-warp shared-memory
+//               transpose and coalesced row stores.
 // Rows beyond M are zero-filled by TMA and never stored.  Requires K % 64 == 0
 // and N % BN == 0 (checked by the launcher).
 #include <cudaTypedefs.h>
