@@ -1,8 +1,9 @@
-// Row-wise HBM-bound kernels on the fp32 residual stream: the routed-token
-// gather (Eq. 8), LayerNorm (the LN of the pre-LN block, Sec. 3.3 Eq. 11) and
-// the conversions between the caller's storage dtype and the stream.  One warp
-// owns one row; rows move as 16-byte vectors, all loads of a row are issued
-// before any use.
+// Row-wise HBM-bound kernels on the fp32 residual stream: LayerNorm (the LN of
+// the pre-LN block, Sec. 3.3 Eq. 11), which for the first sparse block also
+// performs the routed-token gather (Eq. 8) through the index set; the
+// conversions between the caller's storage dtype and the stream; and the fp32
+// sum of an implicit ensemble's members.  One warp owns one row; rows move as
+// 16-byte vectors, all loads of a row are issued before any use.
 #include "common.cuh"
 #include "kernels.h"
 

@@ -7,7 +7,8 @@
 // T and how many keys equal to T must be kept, and an ordered block-wide
 // compaction writes the selected indices, which come out sorted by
 // construction.  Work per sample is O(L * passes); HBM traffic is the index
-// write (4 B per selected token) plus, for the top-K selector, one read of x.
+// write (4 B per selected token) plus, for the top-K selector, the scores: one
+// pass over x computes them, unless the forward's FC2 epilogue already has.
 #include "common.cuh"
 #include "kernels.h"
 
