@@ -28,13 +28,49 @@ if ROOT not in sys.path:
 DEFAULT_WORKLOAD = "c4_0p25deg_bf16"
 L2_FLUSH_BYTES = 512 << 20          # > 129 MB of L2
 
-# DRAM bytes (read + write) per launch of a kernel kind on a workload, from one
-# ncu capture of the current kernel (profiles/attention_tc_c4_*.md): the 0.25 deg
-# forward runs 8 dense attention launches (114.66 MB each) and 16 sparse ones
-# (24.93 MB each).  None when no capture of the current kernel exists.
-DRAM_TRAFFIC_PER_LAUNCH = {
-    ("attention", "c4_0p25deg_bf16"): (8 * 114.66e6 + 16 * 24.93e6) / 24,
+# DRAM bytes (read + write) per launch of a kernel kind, measured by ncu, are
+# kept in a small text table under profiles/ together with a digest of the
+# kernel's source files at the time of the capture.  The roofline reports them
+# only while that digest matches the current sources; otherwise "traffic" is
+# null and a warning names the stale capture.
+TRAFFIC_TABLE = os.path.join(ROOT, "profiles", "dram_traffic_per_launch.txt")
+KERNEL_SOURCES = {
+    "attention": ("attention_tc.cu", "tc_ptx.cuh", "common.cuh", "kernels.h"),
+    "gemm": ("gemm_tc.cu", "tc_ptx.cuh", "common.cuh", "kernels.h"),
 }
+
+
+def source_digest(kind):
+    """sha256 (first 12 hex digits) over the CUDA sources a kernel kind is built from."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES[kind]:
+        with open(os.path.join(ROOT, "paper_2607_02829_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:12]
+
+
+def measured_traffic(kind, workload):
+    """(bytes per launch, note) from the traffic table for this kernel kind and
+    workload, or (None, reason)."""
+    src = "gemm" if kind.startswith("gemm") else kind
+    if src not in KERNEL_SOURCES:
+        return None, f"no ncu traffic figure is kept for {kind}"
+    try:
+        lines = open(TRAFFIC_TABLE).read().splitlines()
+    except OSError:
+        return None, "no traffic table"
+    want = source_digest(src)
+    for line in lines:
+        p = [c.strip() for c in line.strip().strip("|").split("|")]
+        if len(p) >= 4 and p[0] == kind and p[1] == workload:
+            if p[2] != want:
+                msg = (f"the ncu traffic of {kind} on {workload} was captured on sources "
+                       f"{p[2]}, the current ones are {want}: traffic reported as null")
+                print("bench.py: " + msg, file=sys.stderr)
+                return None, msg
+            return float(p[3]) * 1e6, f"ncu capture of sources {p[2]}"
+    return None, f"no ncu traffic figure for {kind} on {workload}"
 
 
 def _peaks():
@@ -252,6 +288,17 @@ def run_ours(args, rank, world, local_rank):
                              + 4.0 * wl.B * K * K * wl.D)
         segment = {"ms": seg_ms, "gflop": seg_flops / 1e9,
                    "tflops": seg_flops / (seg_ms * 1e-3) / 1e12}
+        # the segment traced: every FC2 here runs on the routed rows, so the last
+        # one's extra time over a plain FC2 of the same shape is the scatter's
+        b.sr_trace_enable(senc.handle, True)
+        b.sr_trace_read(senc.handle, reset=True)
+        for i in range(args.steps):
+            flush.zero_()
+            b.sr_forward(senc.handle, x.data_ptr(), sw, wl.keep_ratio, seed + i, out.data_ptr(),
+                         None, stream.cuda_stream)
+        torch.cuda.synchronize()
+        segment["trace"] = b.sr_trace_read(senc.handle, reset=True)
+        b.sr_trace_enable(senc.handle, False)
         senc.close()
 
     # ---- end to end through the C ABI from pinned host memory.  Every step copies
@@ -305,24 +352,35 @@ def run_ours(args, rank, world, local_rank):
 
 
 def roofline(trace, peaks, steps, workload, fp32_alu=False):
+    """The dominant kernel kind of the traced forward against its roofline.  A
+    tensor-bound kind is divided by the burst bf16 peak (its launches last tens
+    to hundreds of microseconds inside a step of about 12 ms); the sustained
+    figure is given beside it."""
     kernels = {k: v for k, v in trace.items() if k != "copy" and v["launches"] > 0}
     dom = max(kernels, key=lambda k: kernels[k]["ms"])
     t = kernels[dom]
     per_launch_ms = t["ms"] / t["launches"]
+    extra = {}
     if t["flops"] > 0 and fp32_alu:
         # CUDA-core fp32 kernels: 152 SMs x 128 FP32 lanes x 2 flops per FFMA at
         # the maximum SM clock
         achieved = t["flops"] / t["launches"] / (per_launch_ms * 1e-3) / 1e12
         peak = 152 * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
         bound, unit = "alu", "TFLOP/s"
+        source = "derived from SM count, FP32 lanes and max clock"
     elif t["flops"] > 0:
         achieved = t["flops"] / t["launches"] / (per_launch_ms * 1e-3) / 1e12
-        peak = peaks["bf16_tflops_sustained"]
+        peak = peaks["bf16_tflops"]
         bound, unit = "tensor", "TFLOP/s"
+        source = peaks["source"] + " burst"
+        extra = {"peak_sustained": peaks["bf16_tflops_sustained"],
+                 "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"]}
     else:
         achieved = t["bytes"] / t["launches"] / (per_launch_ms * 1e-3) / 1e9
         peak = peaks["hbm_gbs"]
         bound, unit = "hbm", "GB/s"
+        source = peaks["source"] + " copy bandwidth"
+    traffic, traffic_note = measured_traffic(dom, workload)
     total_ms = sum(v["ms"] for v in kernels.values())
     detail = {}
     for k, v in kernels.items():
@@ -333,12 +391,42 @@ def roofline(trace, peaks, steps, workload, fp32_alu=False):
         if v["bytes"] > 0:
             d["gbs"] = v["bytes"] / (v["ms"] * 1e-3) / 1e9
         detail[k] = d
-    return ({"kernel": dom, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-             "frac": achieved / peak,
-             "peak_source": ("derived from SM count, FP32 lanes and max clock" if bound == "alu"
-                             else peaks["source"] + (" sustained" if bound == "tensor" else "")),
-             "traffic": DRAM_TRAFFIC_PER_LAUNCH.get((dom, workload)),
-             "algorithmic_bytes_per_launch": t["bytes"] / t["launches"]}, detail)
+    return (dict({"kernel": dom, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+                  "frac": achieved / peak, "peak_source": source}, **extra,
+                 traffic=traffic, traffic_source=traffic_note,
+                 algorithmic_bytes_per_launch=t["bytes"] / t["launches"]), detail)
+
+
+def gather_scatter(wl, K, trace, segment, peaks):
+    """GB/s and fraction of the measured HBM copy bandwidth of the gather (fused
+    into the first sparse LN1) and of the delta scatter (fused into the last
+    sparse FC2), with their algorithmic bytes per launch.
+      gather : the selected fp32 stream rows read, h0 (fp32) and LN1 (storage
+               dtype) written, plus the index set;
+      scatter: x0 rows read and x' rows written (fp32 stream), plus the index
+               set, over the time the scatter FC2 takes beyond a plain FC2 on
+               the same routed rows (both from the sparse segment's trace)."""
+    out = {}
+    g = trace.get("gather", {})
+    if g.get("launches"):
+        gbs = g["bytes"] / (g["ms"] * 1e-3) / 1e9
+        out["gather"] = {"bytes_per_launch": g["bytes"] / g["launches"],
+                         "us_per_launch": g["ms"] / g["launches"] * 1e3,
+                         "gbs": gbs, "frac_of_hbm": gbs / peaks["hbm_gbs"]}
+    st = (segment or {}).get("trace") or {}
+    fs, f = st.get("gemm_fc2_scatter", {}), st.get("gemm_fc2", {})
+    if fs.get("launches") and f.get("launches"):
+        extra_ms = fs["ms"] / fs["launches"] - f["ms"] / f["launches"]
+        nbytes = 8.0 * wl.B * K * wl.D + 4.0 * wl.B * K
+        rec = {"bytes_per_launch": nbytes, "us_fc2_scatter": fs["ms"] / fs["launches"] * 1e3,
+               "us_fc2_plain": f["ms"] / f["launches"] * 1e3}
+        if extra_ms > 0:
+            gbs = nbytes / (extra_ms * 1e-3) / 1e9
+            rec.update(gbs=gbs, frac_of_hbm=gbs / peaks["hbm_gbs"])
+        else:
+            rec["note"] = "the scatter FC2 was not slower than a plain FC2 of the same shape"
+        out["scatter"] = rec
+    return out
 
 
 def cpu_baseline(wl, sparse_only=False):
@@ -392,7 +480,12 @@ def main():
                     help="size sweep of one kernel (prints one JSON line per size)")
     ap.add_argument("--clocks-csv", default=None,
                     help="keep the raw nvidia-smi samples of the timed region in this file")
+    ap.add_argument("--source-digest", choices=sorted(KERNEL_SOURCES), default=None,
+                    help="print the digest of a kernel kind's CUDA sources and exit")
     args = ap.parse_args()
+    if args.source_digest:
+        print(source_digest(args.source_digest))
+        return
     args.warmup = max(args.warmup, 3)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -428,10 +521,9 @@ def main():
     value = job_tokens_per_s(wl.B * wl.L, world, ms)
     roof, detail = roofline(trace, peaks, args.steps, wl.name, fp32_alu=wl.dtype == "f32")
     launches = sum(v["launches"] for v in trace.values())
-    gs = {}
-    for k in ("gather", "gemm_fc2_scatter"):
-        if trace[k]["launches"]:
-            gs[k + "_gbs"] = trace[k]["bytes"] / (trace[k]["ms"] * 1e-3) / 1e9
+    gs = gather_scatter(wl, K, trace, segment, peaks)
+    if segment:
+        segment.pop("trace", None)
     total_flops = sum(v["flops"] for v in trace.values()) / args.steps
     line = {
         "metric": "full-grid tokens/sec of routed encoder fwd",

@@ -191,7 +191,8 @@ sr_status sr_forward_host(sr_handle* h, const void* x_host, const sr_block_weigh
  * event records per launch when on, and records nothing while the stream is
  * being captured into a CUDA graph. */
 typedef enum {
-  SR_KERN_COPY = 0,          /* x -> out device copy when out != x */
+  SR_KERN_COPY = 0,          /* stream conversions and copies: widen x to the fp32
+                                stream, narrow it to out, ensemble sums */
   SR_KERN_SELECT = 1,        /* token selection (and the top-K norms when not fused into FC2) */
   SR_KERN_GATHER = 2,        /* h0 = x[:, I, :] (Eq. 8), fused with LN1 of the first
                                 sparse block: reads the selected rows, writes h0 and LN1 */
@@ -239,9 +240,10 @@ sr_status sr_destroy(sr_handle* h);
  * Returns SR_ERR_UNSUPPORTED when B * L exceeds 1,048,576 (or L or D exceed
  * what the selection kernels support), SR_ERR_INVALID_ARG for bad pointers,
  * dtype or ratio, before any launch.  Calls no cudaMalloc, cudaFree or other
- * allocating routine.  The first call on each device looks up the static
- * array's device address (cudaGetSymbolAddress); make that first call before
- * any stream capture.  All calls share the one array and it keeps the last
+ * allocating routine.  Every call looks up the static array's device address
+ * in the current context (cudaGetSymbolAddress; the first call on a device
+ * also loads the library's module there), so make the first call on each
+ * device before any stream capture.  All calls share the one array and it keeps the last
  * call's scores; each call overwrites every score it reads, so nothing has to
  * start at zero, but calls whose work overlaps on the GPU (other streams, or
  * other host threads on the same device) race on it and must be serialised

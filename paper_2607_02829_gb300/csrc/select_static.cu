@@ -5,7 +5,6 @@
 // static __device__ array instead of a caller-provided workspace.  The array
 // is sized for kStaticScoreTokens tokens (B * L) and stays resident on every
 // GPU that loads this library until the process exits.
-#include <mutex>
 #include <string>
 
 #include "../../include/sparse_reslim.h"
@@ -20,10 +19,6 @@ namespace {
 
 constexpr size_t kStaticScoreTokens = size_t(1) << 20;          // 1,048,576 tokens, 4 MiB
 static __device__ __align__(256) float g_static_scores[kStaticScoreTokens];
-
-constexpr int kMaxDevices = 64;
-float* g_scores_dev[kMaxDevices] = {};                          // device address, per device
-std::mutex g_setup_mu;
 
 // One warp per token: squared L2 norm of the stored row, in the same element
 // order and with the same fp32 accumulation as the workspace path (4 elements
@@ -58,23 +53,17 @@ sr_status reject(sr_status st, const std::string& msg) {
   return st;
 }
 
-// The device address of the static score array on the current device; the
-// first call on each device looks it up (cudaGetSymbolAddress).
+// The device address of the static score array in the current device's context.
+// It is looked up on every call (cudaGetSymbolAddress allocates nothing), so a
+// context that was reset or recreated since an earlier call is never handed a
+// stale address.
 sr_status scores_on_current_device(float** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return reject(SR_ERR_CUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));
-  if (dev < 0 || dev >= kMaxDevices) return reject(SR_ERR_UNSUPPORTED, "device ordinal >= 64");
-  std::lock_guard<std::mutex> lock(g_setup_mu);
-  if (!g_scores_dev[dev]) {
-    float* p = nullptr;
-    e = cudaGetSymbolAddress(reinterpret_cast<void**>(&p), g_static_scores);
-    if (e != cudaSuccess || !p)
-      return reject(SR_ERR_CUDA, std::string("cudaGetSymbolAddress(static scores): ") +
-                                     cudaGetErrorString(e));
-    g_scores_dev[dev] = p;
-  }
-  *out = g_scores_dev[dev];
+  float* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void**>(&p), g_static_scores);
+  if (e != cudaSuccess || !p)
+    return reject(SR_ERR_CUDA, std::string("cudaGetSymbolAddress(static scores): ") +
+                                   cudaGetErrorString(e));
+  *out = p;
   return SR_OK;
 }
 

@@ -39,6 +39,25 @@ def max_norm_rel(y, o):
     return float(np.abs(y - o).max() / max(np.abs(o).max(), 1e-300))
 
 
+# (case, max-norm relative error, 99.9th percentile of |y - o| / max|o|, bar,
+# elements compared), in test order; the session summary prints them
+PARITY_RECORDS = []
+
+
+def check_parity(case, y, o, tol):
+    """Asserts max|y - o| / max|o| <= tol and records that error together with
+    the elementwise 99.9th-percentile error |y - o| / max|o|."""
+    y = np.asarray(y, dtype=np.float64)
+    o = np.asarray(o, dtype=np.float64)
+    scale = max(float(np.abs(o).max()), 1e-300)
+    e = np.abs(y - o).ravel() / scale
+    err = float(e.max())
+    p999 = float(np.quantile(e, 0.999))
+    PARITY_RECORDS.append((case, err, p999, tol, int(e.size)))
+    assert err <= tol, f"{case}: max-norm relative error {err:.3e} exceeds {tol:.0e}"
+    return err
+
+
 def to_device(x, weights):
     xd = x.cuda()
     wd = [{k: v.cuda() for k, v in blk.items()} for blk in weights]

@@ -9,7 +9,7 @@ import torch
 
 from oracle import reslim as o
 from paper_2607_02829_gb300 import synth
-from tests._helpers import built_lib, gpu_forward, max_norm_rel
+from tests._helpers import built_lib, check_parity, gpu_forward
 
 pytestmark = pytest.mark.gpu
 
@@ -147,8 +147,8 @@ def test_forward_parity_small(dtype, B, L, heads, split, r):
     ref, ridx = _oracle(wl, x, ws)
     if r < 1.0:
         assert np.array_equal(idx, ridx)
-    err = max_norm_rel(synth.stored_as_f64(out), ref)
-    assert err <= TOL[dtype], err
+    check_parity(f"small {dtype} B={B} L={L} H={heads} split={split} r={r}",
+                 synth.stored_as_f64(out), ref, TOL[dtype])
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
@@ -182,8 +182,7 @@ def test_forward_parity_workload(wlname):
     out, idx = gpu_forward(wl, x, ws)
     ref, ridx = _oracle(wl, x, ws)
     assert np.array_equal(idx, ridx)
-    err = max_norm_rel(synth.stored_as_f64(out), ref)
-    assert err <= TOL[wl.dtype], err
+    check_parity(f"{wlname} (full output)", synth.stored_as_f64(out), ref, TOL[wl.dtype])
 
 
 # bf16 with D = 128: the scores come from the dense-early block's FC2 epilogue;
@@ -194,8 +193,7 @@ def test_forward_parity_topk_selector_small(dtype, heads):
     x, ws = synth.make_inputs(wl)
     out, idx = gpu_forward(wl, x, ws)
     ref, ridx = _oracle(wl, x, ws, idx=idx)      # same indices on both sides
-    err = max_norm_rel(synth.stored_as_f64(out), ref)
-    assert err <= TOL[dtype], err
+    check_parity(f"small top-K {dtype} H={heads}", synth.stored_as_f64(out), ref, TOL[dtype])
     x0, _ = gpu_forward(wl, x, ws, n_split=(2, 0, 0), want_idx=False)
     assert np.array_equal(idx, o.select_topk_l2(synth.stored_as_f64(x0), 64))
     again, idx2 = gpu_forward(wl, x, ws)
@@ -228,8 +226,8 @@ def test_ensemble_members_bitwise_and_mean(dtype, split, r):
     if r < 1.0:
         for m in range(len(seeds)):
             assert np.array_equal(idx[m].cpu().numpy(), ridx[m])
-    err = max_norm_rel(synth.stored_as_f64(mean.cpu()), ref)
-    assert err <= TOL[dtype], err
+    check_parity(f"ensemble mean {dtype} split={split} r={r}", synth.stored_as_f64(mean.cpu()),
+                 ref, TOL[dtype])
     enc.close()
 
 
@@ -250,8 +248,8 @@ def test_cross_attention_parity(B, Tq, Tkv, heads):
     torch.cuda.synchronize()
     assert int(fault.item()) == 0
     ref = o.cross_attention(synth.stored_as_f64(q), synth.stored_as_f64(kv), heads)
-    err = max_norm_rel(synth.stored_as_f64(out.cpu()), ref)
-    assert err <= TOL["bf16"], err
+    check_parity(f"cross-attention B={B} Tq={Tq} Tkv={Tkv} H={heads}",
+                 synth.stored_as_f64(out.cpu()), ref, TOL["bf16"])
 
 
 def test_cross_attention_routed_over_full_sequence_sampled():
@@ -273,5 +271,4 @@ def test_cross_attention_routed_over_full_sequence_sampled():
     rows = np.concatenate([rows, [0, 255, 256, Tq - 1]])
     ref = o.cross_attention(synth.stored_as_f64(q)[:, rows], synth.stored_as_f64(kv), heads)
     got = synth.stored_as_f64(out.cpu())[:, rows]
-    err = max_norm_rel(got, ref)
-    assert err <= TOL["bf16"], err
+    check_parity("cross-attention 4050 over 16200, 52 sampled rows", got, ref, TOL["bf16"])

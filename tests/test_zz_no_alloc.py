@@ -1,5 +1,5 @@
 """The allocation-free top-K selector (sr_select_topk_l2_static) against the
-workspace-based sr_select.
+fp64 oracle's top-K selection and against the workspace-based sr_select.
 
 Callers that cannot allocate device memory (a plugin inside a framework that
 owns the GPU memory pool and gives it no workspace, or a latency-critical path
@@ -11,6 +11,8 @@ import numpy as np
 import pytest
 import torch
 
+from oracle import reslim as o
+from paper_2607_02829_gb300 import synth
 from tests._helpers import built_lib
 
 pytestmark = pytest.mark.gpu
@@ -57,6 +59,17 @@ def test_static_scratch_topk_matches_workspace_select_twice():
         got = _static_select(b, x, r)
         assert np.array_equal(got, ref)
         assert np.all(np.diff(got, axis=1) > 0)
+        # against the oracle on the same stored values: equal sets, or differences
+        # only inside the fp32 rounding band around the K-th score (the GPU sums
+        # squares in fp32, the oracle in fp64; exact ties are exact on both sides)
+        K = got.shape[1]
+        xf = synth.stored_as_f64(x.cpu())
+        exp = o.select_topk_l2(xf, K)
+        s = o.token_sq_norms(xf)
+        for bb in range(B):
+            kth = np.sort(s[bb])[::-1][K - 1]
+            diff = set(got[bb].tolist()) ^ set(exp[bb].tolist())
+            assert all(abs(s[bb, i] - kth) <= 1e-5 * kth for i in diff), (bb, sorted(diff)[:8])
 
 
 def test_static_scratch_rejects_oversize_before_launch():
