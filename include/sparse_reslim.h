@@ -266,6 +266,32 @@ sr_status sr_device_fault(sr_handle* h, uint32_t* fault, int clear, void* stream
 /* The last CUDA or validation message recorded on this thread ("" if none). */
 const char* sr_last_error_message(void);
 
+/* ---- testing hooks -----------------------------------------------------
+ * The paper has no counterpart of these calls; they exist so that the error
+ * paths can be tested without making a GPU fail. */
+
+/* Host-side fault injection.  From this call on, the CUDA call with index n
+ * (0-based) among those the entry points above make through their checked
+ * path (kernel launches, stream-ordered copies and memsets, stream and event
+ * synchronisation) is not made and reports cudaErrorLaunchFailure instead; the
+ * entry point then returns SR_ERR_CUDA with a message naming the step and
+ * "[injected ...]", and enqueues nothing after it.  n < 0 turns injection off.
+ * Process-wide; resets the count read by sr_debug_enqueue_count. */
+void sr_debug_fail_enqueue(int64_t n);
+
+/* Checked CUDA calls attempted (made, or failed by injection) since the last
+ * sr_debug_fail_enqueue. */
+int64_t sr_debug_enqueue_count(void);
+
+/* Runs the bounded mbarrier wait of the tensor-core kernels on a barrier that
+ * nothing arrives at, with a limit of limit_us microseconds (1 .. 1000000)
+ * instead of the kernels' 2 s: one thread of one CTA waits, gives up, sets bit 0
+ * of *fault (device) as the kernels do, and stores the nanoseconds it waited in
+ * *waited_ns (device).  No TMA or tensor memory is involved; the context stays
+ * usable.  Asynchronous on `stream`. */
+sr_status sr_selftest_wait_timeout(uint32_t* fault, uint32_t limit_us, uint64_t* waited_ns,
+                                   void* stream);
+
 #ifdef __cplusplus
 }
 #endif

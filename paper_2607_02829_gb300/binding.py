@@ -92,6 +92,10 @@ def lib() -> ctypes.CDLL:
         L.sr_select_topk_l2_static.argtypes = [vp, i32, i32, i32, i32, ctypes.c_float, vp,
                                                ctypes.POINTER(i32), vp]
         L.sr_select_topk_l2_static.restype = st
+        L.sr_debug_fail_enqueue.argtypes = [ctypes.c_int64]; L.sr_debug_fail_enqueue.restype = None
+        L.sr_debug_enqueue_count.argtypes = []; L.sr_debug_enqueue_count.restype = ctypes.c_int64
+        L.sr_selftest_wait_timeout.argtypes = [vp, ctypes.c_uint32, vp, vp]
+        L.sr_selftest_wait_timeout.restype = st
         L.sr_status_string.argtypes = [st]; L.sr_status_string.restype = ctypes.c_char_p
         L.sr_last_error_message.argtypes = []; L.sr_last_error_message.restype = ctypes.c_char_p
         _lib = L
@@ -188,6 +192,19 @@ def sr_select_topk_l2_static(x: int, B: int, L: int, D: int, dtype: int, keep_ra
     _check(lib().sr_select_topk_l2_static(x, B, L, D, dtype, keep_ratio, idx, ctypes.byref(K),
                                           stream), "sr_select_topk_l2_static")
     return K.value
+
+
+def sr_debug_fail_enqueue(n: int) -> None:
+    lib().sr_debug_fail_enqueue(int(n))
+
+
+def sr_debug_enqueue_count() -> int:
+    return int(lib().sr_debug_enqueue_count())
+
+
+def sr_selftest_wait_timeout(fault: int, limit_us: int, waited_ns: int, stream: int) -> None:
+    _check(lib().sr_selftest_wait_timeout(fault, limit_us, waited_ns, stream),
+           "sr_selftest_wait_timeout")
 
 
 # ----------------------------------------------------- torch-side helpers

@@ -3,6 +3,7 @@
 // middle -> delta scatter -> dense late).  Everything here is host code; every
 // step of the computation runs in the kernels it launches.
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -29,15 +30,34 @@ sr_status fail(sr_status st, const char* what) {
   return st;
 }
 
+// Host-side fault injection for tests of the error paths: the CUDA call with
+// index g_fail_at (0-based, counted by g_enqueues since the hook was set) is not
+// made and reports cudaErrorLaunchFailure instead.
+std::atomic<long long> g_fail_at{-1};
+std::atomic<long long> g_enqueues{0};
+thread_local bool g_injected = false;
+
+cudaError_t enqueue_gate() {
+  const long long n = g_enqueues.fetch_add(1);
+  g_injected = n == g_fail_at.load();
+  return g_injected ? cudaErrorLaunchFailure : cudaSuccess;
+}
+
 sr_status cuda_fail(cudaError_t e, const char* where) {
-  g_last_msg = std::string(where) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")";
+  g_last_msg = std::string(where) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")" +
+               (g_injected ? " [injected by sr_debug_fail_enqueue]" : "");
+  g_injected = false;
   return SR_ERR_CUDA;
 }
 
-#define SR_CUDA(call, where)                         \
-  do {                                               \
-    cudaError_t e__ = (call);                        \
-    if (e__ != cudaSuccess) return cuda_fail(e__, where); \
+// Every CUDA call of the entry points below goes through the injection gate
+// first; a failed call returns SR_ERR_CUDA at once, so nothing after it is
+// enqueued.
+#define SR_CUDA(call, where)                                \
+  do {                                                      \
+    cudaError_t e__ = enqueue_gate();                       \
+    if (e__ == cudaSuccess) e__ = (call);                   \
+    if (e__ != cudaSuccess) return cuda_fail(e__, where);   \
   } while (0)
 
 constexpr size_t kAlign = 256;
@@ -637,6 +657,13 @@ const char* sr_status_string(sr_status s) {
 }
 
 const char* sr_last_error_message(void) { return g_last_msg.c_str(); }
+
+void sr_debug_fail_enqueue(int64_t n) {
+  g_enqueues.store(0);
+  g_fail_at.store(n < 0 ? -1 : static_cast<long long>(n));
+}
+
+int64_t sr_debug_enqueue_count(void) { return static_cast<int64_t>(g_enqueues.load()); }
 
 sr_status sr_device_fault(sr_handle* h, uint32_t* fault, int clear, void* stream) {
   if (!h || !fault) return fail(SR_ERR_INVALID_ARG, "handle or fault is NULL");

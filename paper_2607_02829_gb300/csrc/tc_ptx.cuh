@@ -55,12 +55,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 // Waits for the phase with the given parity to complete.  Gives up after
-// kWaitLimitNs, or at once when *abort is set by another thread of the CTA; a
-// timeout sets bit 0 of the fault word (in the caller's workspace, read by
-// sr_device_fault) and *abort.  Returns false when it gave up.
+// limit_ns (kWaitLimitNs in the kernels), or at once when *abort is set by
+// another thread of the CTA; a timeout sets bit 0 of the fault word (in the
+// caller's workspace, read by sr_device_fault) and *abort.  Returns false when
+// it gave up.
 template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                          unsigned int* fault) {
+                                          unsigned int* fault,
+                                          unsigned long long limit_ns = kWaitLimitNs) {
   const uint32_t a = smem_u32(bar);
   if (mbar_try_wait<kCluster>(a, parity)) return true;
   const unsigned long long t0 = global_ns();
@@ -68,7 +70,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
     if (mbar_try_wait<kCluster>(a, parity)) return true;
     if ((it & 255u) == 0) {
       if (*abort) return false;
-      if (global_ns() - t0 > kWaitLimitNs) {
+      if (global_ns() - t0 > limit_ns) {
         if (fault) atomicOr(fault, 1u);
         *abort = 1;
         return false;

@@ -273,3 +273,41 @@ def test_static_topk_selector_rejects_arguments_before_any_launch(L):
                                          a["idx"], ctypes.byref(k), None)
         assert got == status, (kw, got)
         assert k.value == -1                                # K_out untouched on a rejection
+
+
+def test_injected_failure_stops_the_forward_at_its_first_call(L):
+    # the host-side injection hook fails the first CUDA call sr_forward would
+    # make: it returns SR_ERR_CUDA with a message naming that step, and attempts
+    # no further call (no GPU is touched: every pointer here is a fake address)
+    from paper_2607_02829_gb300 import binding as b
+    cfg = b.make_config(2, 512, 256, 4, 2, 2, 2, dtype="f32")
+    h = _handle(b, cfg, b.sr_workspace_bytes(cfg, 0.25))
+    try:
+        w = (b.sr_block_weights * 6)()
+        for i in range(6):
+            for f in b.WEIGHT_FIELDS:
+                setattr(w[i], f, 0x200000)
+        b.sr_debug_fail_enqueue(0)
+        with pytest.raises(b.SRError) as e:
+            b.sr_forward(h, 0x400000, w, 0.25, 0, 0x800000, None, None)
+        assert e.value.status == b.SR_ERR_CUDA
+        assert "injected" in str(e.value) and "clear fault word" in str(e.value)
+        assert b.sr_debug_enqueue_count() == 1
+        # an invalid argument is still rejected before any CUDA call is attempted
+        b.sr_debug_fail_enqueue(0)
+        with pytest.raises(b.SRError) as e:
+            b.sr_forward(h, 0x400000, w, 0.0, 0, 0x800000, None, None)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
+        assert b.sr_debug_enqueue_count() == 0
+    finally:
+        b.sr_debug_fail_enqueue(-1)
+        b.sr_destroy(h)
+
+
+def test_selftest_wait_timeout_rejects_bad_arguments(L):
+    from paper_2607_02829_gb300 import binding as b
+    for fault, limit, waited in [(0, 1000, 0x1000), (0x1001, 1000, 0x1000), (0x1000, 0, 0x1000),
+                                 (0x1000, 2000000, 0x1000), (0x1000, 1000, 0), (0x1000, 1000, 0x1004)]:
+        with pytest.raises(b.SRError) as e:
+            b.sr_selftest_wait_timeout(fault, limit, waited, None)
+        assert e.value.status == b.SR_ERR_INVALID_ARG
