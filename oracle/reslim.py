@@ -14,7 +14,9 @@ What it computes (arxiv 2607.02829):
   (the paper draws it with torch.randperm, which cannot be reproduced
   independently; this oracle defines it through SplitMix64 keys, see
   ``random_keys``), and the activation-norm selector of App. B.2 Table 11
-  (top-K by per-token L2 norm of the last dense-early block's output)
+  (top-K by per-token L2 norm of the last dense-early block's output) and the
+  gradient (Laplacian) selector of the same table (top-K by the squared norm
+  of the 5-point Laplacian on the patch grid, see ``token_laplacian_scores``)
 * gather h0 = x[:, I, :] and the sparse middle blocks on h      -- Sec. 3.2 Eq. 8
 * the residual delta and scatter x' = x0 + Scatter(h - h0, I)   -- Sec. 3.2 Eq. 9
 * the pre-LN block h <- h + Attn(LN h); h <- h + MLP(LN h)       -- Sec. 3.3 Eq. 11
@@ -99,6 +101,45 @@ def select_topk_l2(x: np.ndarray, K: int) -> np.ndarray:
     """K tokens with the largest L2 norm per sample (the activation-norm sampler
     of App. B.2 Table 11), ties to the lower token index, sorted ascending."""
     s = token_sq_norms(x)
+    B, L = s.shape
+    out = np.empty((B, K), dtype=np.int64)
+    for b in range(B):
+        order = np.lexsort((np.arange(L), -s[b]))     # primary: -score, secondary: index
+        out[b] = np.sort(order[:K])
+    return out
+
+
+# ------------------------------------- App. B.2: gradient (Laplacian) selector
+def token_laplacian_scores(x: np.ndarray, grid_w: int) -> np.ndarray:
+    """[B, L] Laplacian score of every token (App. B.2 Table 11, "Gradient
+    (Laplacian)"; the paper gives no formula, so this is a reading of it).
+
+    Tokens lie on the patch grid row-major, grid_w tokens per latitude row and
+    L / grid_w rows.  For the token at (i, j), the 5-point Laplacian of its
+    feature vector is
+        lap(i, j) = x(i-1, j) + x(i+1, j) + x(i, j-1) + x(i, j+1) - 4 x(i, j),
+    with longitude periodic (j - 1 and j + 1 wrap around the row) and the first
+    and last latitude rows reflected onto themselves (x(-1, j) = x(0, j),
+    x(H, j) = x(H-1, j): a zero-flux boundary at the poles).  The score is the
+    squared L2 norm over the features, sum_d lap(i, j)_d ** 2."""
+    x = np.asarray(x, dtype=np.float64)
+    B, L, D = x.shape
+    if grid_w < 1 or L % grid_w != 0:
+        raise ValueError("L must be a multiple of grid_w")
+    H = L // grid_w
+    g = x.reshape(B, H, grid_w, D)
+    north = np.concatenate([g[:, :1], g[:, :-1]], axis=1)       # x(i-1, j), row 0 reflected
+    south = np.concatenate([g[:, 1:], g[:, -1:]], axis=1)       # x(i+1, j), row H-1 reflected
+    west = np.roll(g, 1, axis=2)                                 # x(i, j-1), periodic
+    east = np.roll(g, -1, axis=2)                                # x(i, j+1), periodic
+    lap = north + south + west + east - 4.0 * g
+    return np.einsum("bhwd,bhwd->bhw", lap, lap).reshape(B, L)
+
+
+def select_topk_laplacian(x: np.ndarray, K: int, grid_w: int) -> np.ndarray:
+    """K tokens with the largest Laplacian score per sample, ties to the lower
+    token index, sorted ascending (the gradient-based sampler of App. B.2)."""
+    s = token_laplacian_scores(x, grid_w)
     B, L = s.shape
     out = np.empty((B, K), dtype=np.int64)
     for b in range(B):
@@ -222,7 +263,7 @@ def forward(x: np.ndarray, weights: Sequence[Dict[str, np.ndarray]], n1: int, n2
             n3: int, heads: int, keep_ratio: float, seed: int = 0,
             selector: str = "random", shared_indices: bool = False, eps: float = 1e-5,
             idx: Optional[np.ndarray] = None, bypass_dense: bool = True,
-            threads: int = 0, return_stages: bool = False):
+            threads: int = 0, return_stages: bool = False, grid_w: int = 0):
     """The routed encoder of Alg. 1 (dense early, sparse middle, dense late) in fp64.
 
     x: [B, L, D]; weights: N = n1 + n2 + n3 dicts of block weights.
@@ -249,6 +290,8 @@ def forward(x: np.ndarray, weights: Sequence[Dict[str, np.ndarray]], n1: int, n2
                 idx = select_random(B, L, K, seed, shared_indices)
             elif selector == "topk_l2":
                 idx = select_topk_l2(x, K)
+            elif selector == "laplacian":
+                idx = select_topk_laplacian(x, K, grid_w)
             else:
                 raise ValueError(selector)
         if routed:
@@ -277,7 +320,7 @@ def forward(x: np.ndarray, weights: Sequence[Dict[str, np.ndarray]], n1: int, n2
 def forward_ensemble(x: np.ndarray, weights: Sequence[Dict[str, np.ndarray]], n1: int, n2: int,
                      n3: int, heads: int, keep_ratio: float, seeds: Sequence[int],
                      selector: str = "random", shared_indices: bool = False, eps: float = 1e-5,
-                     threads: int = 0):
+                     threads: int = 0, grid_w: int = 0):
     """Implicit ensembling (Sec. 3, "Training and inference"; App. B): the mean
     of the routed forward over a set of selection seeds, each member a plain
     call of ``forward``.  Returns (mean, [member outputs], [member index sets]).
@@ -285,7 +328,7 @@ def forward_ensemble(x: np.ndarray, weights: Sequence[Dict[str, np.ndarray]], n1
     outs, idxs = [], []
     for seed in seeds:
         y, idx = forward(x, weights, n1, n2, n3, heads, keep_ratio, seed=seed, selector=selector,
-                         shared_indices=shared_indices, eps=eps, threads=threads)
+                         shared_indices=shared_indices, eps=eps, threads=threads, grid_w=grid_w)
         outs.append(y)
         idxs.append(idx)
     return sum(outs) / float(len(outs)), outs, idxs

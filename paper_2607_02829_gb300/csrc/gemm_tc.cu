@@ -18,7 +18,9 @@
 //               swizzled shared-memory tiles; the fp32 residual is updated by
 //               TMA reduce (bias + accumulator added into the stream in L2);
 //               the scatter and 64-column tiles use a per-warp shared-memory
-//               transpose and coalesced row stores.
+//               transpose and coalesced row stores (the scatter's rows are
+//               prefetched into L2 during the mainloop and loaded one step
+//               ahead).
 // Rows beyond M are zero-filled by TMA and never stored.  Requires K % 64 == 0
 // and N % BN == 0 (checked by the launcher).
 #include <cudaTypedefs.h>
@@ -101,6 +103,10 @@ __device__ __forceinline__ void gelu2_as7126(float& z0, float& z1) {
   up2(mul2(mul2(mul2(t, poly), pk2(ex2(a0), ex2(a1))), pk2(0.5f, 0.5f)), h0, h1);
   const uint64_t phi = pk2(z0 >= 0.f ? 1.0f - h0 : h0, z1 >= 0.f ? 1.0f - h1 : h1);
   up2(mul2(pk2(z0, z1), phi), z0, z1);
+}
+
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
 }
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
@@ -565,6 +571,77 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           __syncwarp();
           break;
         }
+        }
+      } else if constexpr (E == Epi::BiasResidualScatter) {
+        // last sparse block: hn = h + f(h); x'[xrow] = x0 + (hn - x0), h0 == x0.
+        // The warp walks its 32 rows x BN/2 columns in steps of 16 rows x 32
+        // columns.  A step's global loads (the routed rows h and the stream rows
+        // x0 they scatter into, 128 contiguous bytes per row) are issued one step
+        // ahead, the first step's before the accumulator is ready, so a step waits
+        // for at most one round trip and its stores overlap the next step's
+        // loads.  Element offsets fit 32 bits: sr_create rejects B * L * width
+        // >= 2^31.
+        constexpr int kSteps = 2 * (BN / 64);
+        const int m_lane = row0 + lane;
+        const uint32_t xrow_lane =
+            m_lane < M ? (uint32_t(m_lane / ea.Kr) * uint32_t(ea.Lx) + uint32_t(__ldg(ea.idx + m_lane))) *
+                             uint32_t(N)
+                       : 0u;
+        const float* hres = ea.res;
+        float* xs = static_cast<float*>(ea.out);
+        // step st: columns c_begin + 32 (st / 2) .. + 31, rows 16 (st % 2) .. + 15
+        auto load_step = [&](int st, float (&h)[16], float (&x)[16]) {
+          const int n = nt * BN + c_begin + 32 * (st >> 1) + lane;
+          const int i0 = 16 * (st & 1);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const uint32_t xr = __shfl_sync(0xffffffffu, xrow_lane, i0 + i);
+            const bool v = row0 + i0 + i < M;
+            h[i] = v ? hres[size_t(row0 + i0 + i) * N + n] : 0.f;
+            x[i] = v ? xs[xr + uint32_t(n)] : 0.f;
+          }
+        };
+        // every row this warp reads moves into L2 while the tile's mainloop runs
+        if (m_lane < M) {
+          const char* hp = reinterpret_cast<const char*>(hres + size_t(m_lane) * N + nt * BN + c_begin);
+          const char* xp = reinterpret_cast<const char*>(xs + xrow_lane + uint32_t(nt * BN + c_begin));
+#pragma unroll
+          for (int l = 0; l < BN / 2 * 4 / 128; ++l) {
+            prefetch_l2(hp + 128 * l);
+            prefetch_l2(xp + 128 * l);
+          }
+        }
+        float rv[2][16], x0[2][16];
+        load_step(0, rv[0], x0[0]);
+        if (!__all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault))) break;
+        tc_fence_after();
+        const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
+        float* stg = staging + (warp - 2) * C::kStageFloats;
+#pragma unroll
+        for (int st = 0; st < kSteps; ++st) {
+          const int c = c_begin + 32 * (st >> 1);
+          if ((st & 1) == 0) {
+            // this thread's row of the chunk's accumulators into the transpose buffer
+            uint32_t r[32];
+            tmem_ld32(tbase + uint32_t(c), r);
+            tmem_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 32; ++j) stg[lane * 33 + j] = __uint_as_float(r[j]);
+            __syncwarp();
+          }
+          if (st + 1 < kSteps) load_step(st + 1, rv[(st + 1) & 1], x0[(st + 1) & 1]);
+          const int col = nt * BN + c + lane;
+          const float bias = __bfloat162float(static_cast<const bf16*>(ea.bias)[col]);
+          const int i0 = 16 * (st & 1);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const uint32_t xr = __shfl_sync(0xffffffffu, xrow_lane, i0 + i);
+            if (row0 + i0 + i < M) {
+              const float hn = rv[st & 1][i] + (stg[(i0 + i) * 33 + lane] + bias);
+              xs[xr + uint32_t(col)] = x0[st & 1][i] + (hn - x0[st & 1][i]);
+            }
+          }
+          if (st & 1) __syncwarp();      // the next chunk rewrites the transpose buffer
         }
       } else {
         // the first chunk's residual loads overlap the wait for the accumulator

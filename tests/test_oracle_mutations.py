@@ -77,6 +77,59 @@ def m_topk_smallest(x, K):
     return out
 
 
+def _lap(x, grid_w, *, lat="reflect", lon="periodic", centre=4.0, transpose=False):
+    x = np.asarray(x, dtype=np.float64)
+    B, L, D = x.shape
+    H = L // grid_w
+    g = x.reshape(B, grid_w, H, D).transpose(0, 2, 1, 3) if transpose else x.reshape(B, H, grid_w, D)
+    if lat == "reflect":
+        north = np.concatenate([g[:, :1], g[:, :-1]], axis=1)
+        south = np.concatenate([g[:, 1:], g[:, -1:]], axis=1)
+    elif lat == "periodic":
+        north, south = np.roll(g, 1, axis=1), np.roll(g, -1, axis=1)
+    else:                                      # zero outside the grid
+        z = np.zeros_like(g[:, :1])
+        north = np.concatenate([z, g[:, :-1]], axis=1)
+        south = np.concatenate([g[:, 1:], z], axis=1)
+    if lon == "periodic":
+        west, east = np.roll(g, 1, axis=2), np.roll(g, -1, axis=2)
+    else:                                      # reflected at the first and last column
+        west = np.concatenate([g[:, :, :1], g[:, :, :-1]], axis=2)
+        east = np.concatenate([g[:, :, 1:], g[:, :, -1:]], axis=2)
+    lap = north + south + west + east - centre * g
+    s = np.einsum("bhwd,bhwd->bhw", lap, lap)
+    return (s.transpose(0, 2, 1) if transpose else s).reshape(B, L)
+
+
+def m_lap_lat_periodic(x, grid_w):
+    return _lap(x, grid_w, lat="periodic")
+
+
+def m_lap_lat_zero(x, grid_w):
+    return _lap(x, grid_w, lat="zero")
+
+
+def m_lap_lon_reflected(x, grid_w):
+    return _lap(x, grid_w, lon="reflect")
+
+
+def m_lap_centre_two(x, grid_w):
+    return _lap(x, grid_w, centre=2.0)
+
+
+def m_lap_grid_transposed(x, grid_w):
+    return _lap(x, grid_w, transpose=True)
+
+
+def m_lap_topk_ties_high(x, K, grid_w):
+    s = o.token_laplacian_scores(x, grid_w)
+    B, L = s.shape
+    out = np.empty((B, K), dtype=np.int64)
+    for b in range(B):
+        out[b] = np.sort(np.lexsort((-np.arange(L), -s[b]))[:K])
+    return out
+
+
 def m_ln_unbiased(v, g, b, eps):
     mu = v.mean(axis=-1, keepdims=True)
     var = v.var(axis=-1, ddof=1, keepdims=True)
@@ -166,7 +219,7 @@ def m_block_no_mlp_residual(x, w, heads, eps=1e-5, pool=None):
 
 def _routed_forward(x, weights, n1, n2, n3, heads, keep_ratio, seed=0, selector="random",
                     shared_indices=False, eps=1e-5, idx=None, bypass_dense=True, threads=0,
-                    return_stages=False, *, scatter_sample0=False, no_gather=False,
+                    return_stages=False, grid_w=0, *, scatter_sample0=False, no_gather=False,
                     skip_late=False, topk_on_input=False):
     x_in = np.asarray(x, dtype=np.float64)
     x = x_in
@@ -177,8 +230,10 @@ def _routed_forward(x, weights, n1, n2, n3, heads, keep_ratio, seed=0, selector=
     routed = n2 > 0 and not (keep_ratio == 1.0 and bypass_dense)
     if idx is None and routed:
         K = o.keep_count(L, keep_ratio)
+        xs = x_in if topk_on_input else x
         idx = (o.select_random(B, L, K, seed, shared_indices) if selector == "random"
-               else o.select_topk_l2(x_in if topk_on_input else x, K))
+               else o.select_topk_laplacian(xs, K, grid_w) if selector == "laplacian"
+               else o.select_topk_l2(xs, K))
     if routed:
         bsel = np.zeros((B, 1), dtype=np.int64) if scatter_sample0 else np.arange(B)[:, None]
         if no_gather:
@@ -256,6 +311,18 @@ CASES = [
      ["test_topk_bruteforce_with_ties"]),
     ("top-K keeps the smallest norms", {"select_topk_l2": m_topk_smallest},
      ["test_topk_bruteforce_with_ties"]),
+    ("Laplacian: latitude wraps around", {"token_laplacian_scores": m_lap_lat_periodic},
+     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce"]),
+    ("Laplacian: zero outside the poles", {"token_laplacian_scores": m_lap_lat_zero},
+     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce"]),
+    ("Laplacian: longitude reflected, not periodic", {"token_laplacian_scores": m_lap_lon_reflected},
+     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce"]),
+    ("Laplacian: centre weight 2", {"token_laplacian_scores": m_lap_centre_two},
+     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce"]),
+    ("Laplacian: grid rows and columns swapped", {"token_laplacian_scores": m_lap_grid_transposed},
+     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce"]),
+    ("Laplacian top-K ties to the higher index", {"select_topk_laplacian": m_lap_topk_ties_high},
+     ["test_laplacian_topk_bruteforce_with_ties"]),
     ("LayerNorm with the unbiased variance", {"layer_norm": m_ln_unbiased},
      ["test_layer_norm_closed_form_and_torch"]),
     ("LayerNorm eps outside the square root", {"layer_norm": m_ln_eps_outside},
@@ -286,7 +353,8 @@ CASES = [
     ("dense-late blocks skipped", {"forward": _fwd_variant(skip_late=True)},
      ["test_r1_is_exactly_the_dense_stack", "test_zero_routed_blocks_leave_everything_bitwise"]),
     ("top-K scored on the input, not the block-n1 output", {"forward": _fwd_variant(topk_on_input=True)},
-     ["test_topk_selector_in_forward_uses_post_dense_state"]),
+     ["test_topk_selector_in_forward_uses_post_dense_state",
+      "test_laplacian_selector_in_forward_uses_post_dense_state"]),
     ("cross-attention with k and v swapped", {"cross_attention": m_cross_kv_swapped},
      ["test_cross_attention_against_torch_sdpa_and_bruteforce",
       "test_cross_attention_single_key_returns_its_value"]),
@@ -337,7 +405,8 @@ CONTROLS = [
      ["test_unselected_tokens_keep_pre_routing_values_exactly",
       "test_routed_block_equals_block_on_extracted_subsequence", "test_r1_is_exactly_the_dense_stack",
       "test_zero_routed_blocks_leave_everything_bitwise",
-      "test_topk_selector_in_forward_uses_post_dense_state"]),
+      "test_topk_selector_in_forward_uses_post_dense_state",
+      "test_laplacian_selector_in_forward_uses_post_dense_state"]),
     ("cross-attention restatement", {"cross_attention": lambda q, kv, heads, pool=None: _cross(q, kv, heads)},
      ["test_cross_attention_against_torch_sdpa_and_bruteforce",
       "test_cross_attention_single_key_returns_its_value",

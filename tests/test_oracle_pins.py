@@ -127,6 +127,68 @@ def test_topk_bruteforce_with_ties():
             assert idx[b].tolist() == sorted(order[:K])
 
 
+# ----------------------------------------- Laplacian selector (App. B.2)
+def _lap_scores_bruteforce(x, grid_w):
+    """Pure-Python 5-point Laplacian score: clamp the latitude index to the grid
+    (the poles reflected onto themselves), wrap the longitude index."""
+    B, L, D = x.shape
+    H = L // grid_w
+    s = np.zeros((B, L))
+    for b in range(B):
+        for i in range(H):
+            for j in range(grid_w):
+                def at(ii, jj):
+                    return x[b, min(max(ii, 0), H - 1) * grid_w + jj % grid_w]
+                lap = at(i - 1, j) + at(i + 1, j) + at(i, j - 1) + at(i, j + 1) - 4.0 * at(i, j)
+                s[b, i * grid_w + j] = sum(float(v) * float(v) for v in lap)
+    return s
+
+
+def test_laplacian_scores_closed_forms():
+    H, W, D = 6, 8, 3
+    a = np.array([0.5, -1.25, 2.0])
+    # a constant field has no curvature
+    assert np.all(o.token_laplacian_scores(np.full((2, H * W, D), 3.7), W) == 0.0)
+    # quadratic in latitude, x = a i^2: interior rows 4 |a|^2; the first row
+    # sees x(1) - x(0) = a, the last x(H-2) - x(H-1) = -(2H - 3) a
+    i = np.repeat(np.arange(H), W).astype(np.float64)
+    x = (i[:, None] ** 2 * a[None, :])[None]
+    s = o.token_laplacian_scores(x, W).reshape(H, W)
+    na = float(np.dot(a, a))
+    assert np.allclose(s[1:-1], 4.0 * na, rtol=0, atol=1e-12)
+    assert np.allclose(s[0], na, rtol=0, atol=1e-12)
+    assert np.allclose(s[-1], (2 * H - 3) ** 2 * na, rtol=0, atol=1e-9)
+    # a longitude wave, x = c cos(2 pi k j / W), is an eigenfunction of the
+    # periodic second difference: lap = 2 (cos(2 pi k / W) - 1) x
+    for k in (1, 3):
+        j = np.tile(np.arange(W), H).astype(np.float64)
+        c = np.array([1.0, -0.5, 0.25])
+        cw = np.cos(2 * np.pi * k * j / W)
+        x = (cw[:, None] * c[None, :])[None]
+        expect = 4.0 * (np.cos(2 * np.pi * k / W) - 1.0) ** 2 * cw ** 2 * float(np.dot(c, c))
+        assert np.allclose(o.token_laplacian_scores(x, W)[0], expect, rtol=0, atol=1e-12)
+
+
+def test_laplacian_scores_bruteforce():
+    rng = np.random.default_rng(11)
+    for (B, H, W, D) in [(2, 5, 7, 4), (1, 1, 6, 3), (1, 4, 1, 2), (3, 3, 3, 5)]:
+        x = rng.standard_normal((B, H * W, D))
+        assert np.allclose(o.token_laplacian_scores(x, W), _lap_scores_bruteforce(x, W),
+                           rtol=1e-13, atol=1e-13)
+
+
+def test_laplacian_topk_bruteforce_with_ties():
+    rng = np.random.default_rng(5)
+    H, W = 4, 5
+    x = rng.integers(-1, 2, size=(2, H * W, 3)).astype(np.float64)   # many equal scores
+    s = _lap_scores_bruteforce(x, W)
+    for K in (1, 4, 9, 20):
+        idx = o.select_topk_laplacian(x, K, W)
+        for b in range(2):
+            order = sorted(range(H * W), key=lambda t: (-s[b, t], t))
+            assert idx[b].tolist() == sorted(order[:K])
+
+
 # ---------------------------------------------------- block ingredients
 def test_layer_norm_closed_form_and_torch():
     v = np.array([1.0, 2.0, 3.0, 4.0])
@@ -301,6 +363,13 @@ def test_topk_selector_in_forward_uses_post_dense_state():
     out, idx, x0 = o.forward(x, ws, 1, 1, 1, heads=2, keep_ratio=0.25, selector="topk_l2",
                              return_stages=True)
     assert np.array_equal(idx, o.select_topk_l2(x0, 6))
+
+
+def test_laplacian_selector_in_forward_uses_post_dense_state():
+    x, ws = _tiny_model(N=3)                 # L = 24 tokens on a 6 x 4 patch grid
+    out, idx, x0 = o.forward(x, ws, 1, 1, 1, heads=2, keep_ratio=0.25, selector="laplacian",
+                             return_stages=True, grid_w=4)
+    assert np.array_equal(idx, o.select_topk_laplacian(x0, 6, 4))
 
 
 # ------------------------------------------------------------------ implicit ensemble
