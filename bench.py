@@ -208,7 +208,7 @@ def run_ours(args, rank, world, local_rank):
     wl = _workload(args.workload, args.split)
     K = b.sr_keep_count(wl.L, wl.keep_ratio)
     cfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, wl.n1, wl.n2, wl.n3, dtype=wl.dtype,
-                        selector=wl.selector)
+                        selector=wl.selector, grid_w=wl.grid_wp)
     enc = b.Encoder(cfg, max_keep_ratio=wl.keep_ratio)
     # each rank: its own batch (seeded by rank), shared weights
     x_cpu, w_cpu = rank_inputs(wl, rank)
@@ -267,7 +267,7 @@ def run_ours(args, rank, world, local_rank):
     segment = None
     if wl.n2 > 0 and wl.keep_ratio < 1.0:
         scfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, 0, wl.n2, 0, dtype=wl.dtype,
-                             selector=wl.selector)
+                             selector=wl.selector, grid_w=wl.grid_wp)
         senc = b.Encoder(scfg, max_keep_ratio=wl.keep_ratio)
         sw = b.weights_array(wd[wl.n1:wl.n1 + wl.n2])
         for i in range(args.warmup):
@@ -610,7 +610,7 @@ def ensemble_sweep(args):
     wl = _workload(args.workload, args.split)
     x, ws = rank_inputs(wl, 0)
     cfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, wl.n1, wl.n2, wl.n3, dtype=wl.dtype,
-                        selector=wl.selector)
+                        selector=wl.selector, grid_w=wl.grid_wp)
     enc = b.Encoder(cfg, max_keep_ratio=wl.keep_ratio)
     xd = x.cuda()
     warr = b.weights_array([{k: v.cuda() for k, v in blk.items()} for blk in ws])

@@ -60,8 +60,20 @@ typedef enum { SR_F32 = 0, SR_BF16 = 1 } sr_dtype;
  *                  sr_forward with bf16 storage, n1 >= 1 and D % 128 == 0 the
  *                  norms come out of the last dense-early block's FC2
  *                  epilogue; otherwise (and always in sr_select) a separate
- *                  pass reads the stream. */
-typedef enum { SR_SEL_RANDOM = 0, SR_SEL_TOPK_L2 = 1 } sr_selector;
+ *                  pass reads the stream.
+ *  SR_SEL_LAPLACIAN: the K tokens with the largest Laplacian score of the
+ *                  last dense-early block's output (the gradient-based
+ *                  sampler of App. B.2, Table 11, which gives no formula; this
+ *                  library reads it as follows).  Tokens lie row-major on the
+ *                  patch grid, grid_w per latitude row; the score of token
+ *                  (i, j) is the squared L2 norm over D of the 5-point
+ *                  Laplacian x(i-1,j) + x(i+1,j) + x(i,j-1) + x(i,j+1) -
+ *                  4 x(i,j), with longitude periodic and the first and last
+ *                  latitude rows reflected onto themselves (x(-1,j) = x(0,j),
+ *                  x(H,j) = x(H-1,j)).  Values are rounded to the storage
+ *                  dtype first and the score is accumulated in fp32; ties go
+ *                  to the lower token index. */
+typedef enum { SR_SEL_RANDOM = 0, SR_SEL_TOPK_L2 = 1, SR_SEL_LAPLACIAN = 2 } sr_selector;
 
 typedef struct {
   int32_t B;              /* batch size, >= 1 */
@@ -75,6 +87,8 @@ typedef struct {
   int32_t shared_indices; /* 0: one index set per sample (Sec. 3.2 text);
                              1: one set for the whole batch (App. A.4 listing) */
   float ln_eps;           /* LayerNorm epsilon, > 0 (PyTorch's default is 1e-5) */
+  int32_t grid_w;         /* tokens per latitude row of the patch grid; L % grid_w == 0.
+                             Read by SR_SEL_LAPLACIAN only (0 otherwise) */
 } sr_config;
 
 /* Device pointers of one pre-LN block (Sec. 3.3 Eq. 11), nn.Linear layout
@@ -106,13 +120,13 @@ size_t sr_workspace_bytes(const sr_config* cfg, float max_keep_ratio);
 sr_status sr_create(const sr_config* cfg, void* workspace, size_t ws_bytes, sr_handle** out);
 
 /* Token selection alone (Sec. 3.2 / App. B.2).
- *  x      : [B, L, D] device; read only by SR_SEL_TOPK_L2 (the tensor the
- *           norms are taken of), may be NULL for SR_SEL_RANDOM.
+ *  x      : [B, L, D] device; read only by SR_SEL_TOPK_L2 and SR_SEL_LAPLACIAN
+ *           (the tensor the scores are taken of), may be NULL for SR_SEL_RANDOM.
  *  idx    : [B, K] int32 device output, each row strictly increasing.
  *  K_out  : host int32, receives K (may be NULL).
  * Returns SR_ERR_INVALID_ARG when keep_ratio is outside (0, 1] or K < 1.
- * The top-K selector uses the workspace for its per-token scores; the random
- * selector touches only idx. */
+ * The score-based selectors use the workspace for their per-token scores; the
+ * random selector touches only idx. */
 sr_status sr_select(sr_handle* h, const void* x, float keep_ratio, uint64_t seed,
                     int32_t* idx, int32_t* K_out, void* stream);
 
@@ -127,7 +141,8 @@ sr_status sr_select(sr_handle* h, const void* x, float keep_ratio, uint64_t seed
  *            the same arguments.  SR_SEL_TOPK_L2 ranks the output of the last
  *            dense-early block (x itself when n1 == 0); sr_select given that
  *            tensor picks the same set up to ties of the fp32 scores (the
- *            sums are added in a different order).
+ *            sums are added in a different order).  SR_SEL_LAPLACIAN ranks
+ *            the same tensor, with the same scores as sr_select.
  * keep_ratio == 1 runs the plain dense stack (Sec. 3.4, "Architecture-agnostic design": r = 1 is the dense
  * baseline), with no selection, gather or scatter; n2 == 0 likewise routes
  * nothing.  Unselected rows of out are bit-identical to the input of the first
@@ -139,19 +154,28 @@ sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, flo
 /* Implicit ensemble (Sec. 3, "Training and inference"; App. B): averaging the
  * outputs of forward passes with different selection seeds.  Member m is
  * exactly sr_forward(x, seeds[m]); the n1 dense-early blocks do not depend on
- * the seed, so they run once and their result is reused by every member.
+ * the seed, so they run once (on the handle) and their result is copied to
+ * every member.  The members' selection uses the handle; their sparse-middle
+ * and dense-late blocks run together as one batch of M * B samples in the
+ * ensemble workspace (member m's sample b is sample m * B + b), one launch
+ * sequence for all members.  When nothing is routed (keep_ratio == 1 or
+ * n2 == 0) every member is the same dense forward, which runs once and is the
+ * mean.
  *  seeds        : HOST array of M >= 1 selection seeds.
- *  ens_workspace: device buffer of at least sr_ensemble_workspace_bytes(cfg)
- *                 bytes, 256-byte aligned, caller-owned (the dense-early result
- *                 and the fp32 sum of the members).
+ *  ens_workspace: device buffer of at least sr_ensemble_workspace_bytes(cfg, M,
+ *                 keep_ratio) bytes, 256-byte aligned, caller-owned (the
+ *                 batch's fp32 stream and per-block buffers: the workspace of a
+ *                 config with M * B samples).
  *  out          : [B, L, D] device; the mean over the members of their fp32
  *                 results, rounded once to the storage dtype.  May equal x.
  *  members_out  : optional [M, B, L, D] device; member m's output, bit-identical
  *                 to sr_forward's for seed seeds[m].  NULL to skip.
  *  idx_out      : optional [M, B, K] int32 device; member m's index set.
- * Errors as sr_forward, plus SR_ERR_INVALID_ARG for M < 1 or NULL seeds and
- * SR_ERR_WORKSPACE for a missing or short ensemble workspace. */
-size_t sr_ensemble_workspace_bytes(const sr_config* cfg);
+ * Errors as sr_forward, plus SR_ERR_INVALID_ARG for M < 1 or NULL seeds,
+ * SR_ERR_UNSUPPORTED when the batch of M * B samples exceeds what the kernels
+ * accept, and SR_ERR_WORKSPACE for a missing or short ensemble workspace.
+ * sr_ensemble_workspace_bytes returns 0 for an invalid config or M < 1. */
+size_t sr_ensemble_workspace_bytes(const sr_config* cfg, int32_t M, float max_keep_ratio);
 sr_status sr_forward_ensemble(sr_handle* h, const void* x, const sr_block_weights* w,
                               float keep_ratio, const uint64_t* seeds, int32_t M,
                               void* ens_workspace, size_t ens_ws_bytes, void* out,

@@ -16,7 +16,7 @@ LIB_PATH = os.path.join(PKG, "libsparse_reslim.so")
 
 SR_OK, SR_ERR_INVALID_ARG, SR_ERR_UNSUPPORTED, SR_ERR_WORKSPACE, SR_ERR_CUDA, SR_ERR_INTERNAL = range(6)
 SR_F32, SR_BF16 = 0, 1
-SR_SEL_RANDOM, SR_SEL_TOPK_L2 = 0, 1
+SR_SEL_RANDOM, SR_SEL_TOPK_L2, SR_SEL_LAPLACIAN = 0, 1, 2
 
 KERNEL_KINDS = ("copy", "select", "gather", "layernorm", "gemm_qkv", "attention", "gemm_out",
                 "gemm_fc1", "gemm_fc2", "gemm_fc2_scatter")
@@ -27,7 +27,8 @@ class sr_config(ctypes.Structure):
                 ("heads", ctypes.c_int32), ("mlp_hidden", ctypes.c_int32),
                 ("n1", ctypes.c_int32), ("n2", ctypes.c_int32), ("n3", ctypes.c_int32),
                 ("dtype", ctypes.c_int32), ("selector", ctypes.c_int32),
-                ("shared_indices", ctypes.c_int32), ("ln_eps", ctypes.c_float)]
+                ("shared_indices", ctypes.c_int32), ("ln_eps", ctypes.c_float),
+                ("grid_w", ctypes.c_int32)]
 
 
 WEIGHT_FIELDS = ("ln1_g", "ln1_b", "wqkv", "bqkv", "wo", "bo",
@@ -75,7 +76,7 @@ def lib() -> ctypes.CDLL:
         L.sr_forward_host.argtypes = [vp, vp, ctypes.POINTER(sr_block_weights), ctypes.c_float,
                                       ctypes.c_uint64, vp, vp, vp, vp]
         L.sr_forward_host.restype = st
-        L.sr_ensemble_workspace_bytes.argtypes = [ctypes.POINTER(sr_config)]
+        L.sr_ensemble_workspace_bytes.argtypes = [ctypes.POINTER(sr_config), i32, ctypes.c_float]
         L.sr_ensemble_workspace_bytes.restype = sz
         L.sr_forward_ensemble.argtypes = [vp, vp, ctypes.POINTER(sr_block_weights), ctypes.c_float,
                                           ctypes.POINTER(ctypes.c_uint64), i32, vp, sz, vp, vp, vp,
@@ -144,8 +145,8 @@ def sr_forward_host(handle: int, x_host: int, weights: ctypes.Array, keep_ratio:
                                  out_host, idx_out, stream), "sr_forward_host")
 
 
-def sr_ensemble_workspace_bytes(cfg: sr_config) -> int:
-    return int(lib().sr_ensemble_workspace_bytes(ctypes.byref(cfg)))
+def sr_ensemble_workspace_bytes(cfg: sr_config, M: int, max_keep_ratio: float) -> int:
+    return int(lib().sr_ensemble_workspace_bytes(ctypes.byref(cfg), M, max_keep_ratio))
 
 
 def sr_forward_ensemble(handle: int, x: int, weights: ctypes.Array, keep_ratio: float,
@@ -209,11 +210,12 @@ def sr_selftest_wait_timeout(fault: int, limit_us: int, waited_ns: int, stream: 
 
 # ----------------------------------------------------- torch-side helpers
 def make_config(B, L, D, heads, n1, n2, n3, dtype="bf16", selector="random", shared=False,
-                mlp_hidden=None, ln_eps=1e-5) -> sr_config:
+                mlp_hidden=None, ln_eps=1e-5, grid_w=0) -> sr_config:
     return sr_config(B=B, L=L, D=D, heads=heads, mlp_hidden=mlp_hidden or 4 * D, n1=n1, n2=n2,
                      n3=n3, dtype={"f32": SR_F32, "bf16": SR_BF16}[dtype],
-                     selector={"random": SR_SEL_RANDOM, "topk_l2": SR_SEL_TOPK_L2}[selector],
-                     shared_indices=int(bool(shared)), ln_eps=ln_eps)
+                     selector={"random": SR_SEL_RANDOM, "topk_l2": SR_SEL_TOPK_L2,
+                               "laplacian": SR_SEL_LAPLACIAN}[selector],
+                     shared_indices=int(bool(shared)), ln_eps=ln_eps, grid_w=grid_w)
 
 
 def weights_array(blocks: Sequence[dict]) -> ctypes.Array:
@@ -282,7 +284,9 @@ class Encoder:
         (out, members [M, B, L, D] or None, idx [M, B, K] or None)."""
         import torch
         M = len(seeds)
-        nbytes = sr_ensemble_workspace_bytes(self.cfg)
+        nbytes = sr_ensemble_workspace_bytes(self.cfg, M, keep_ratio)
+        if nbytes == 0:
+            raise SRError(SR_ERR_INVALID_ARG, "invalid ensemble: " + lib().sr_last_error_message().decode())
         if getattr(self, "ens_ws", None) is None or self.ens_ws.numel() < nbytes + 256:
             self.ens_ws = torch.empty(nbytes + 256, dtype=torch.uint8, device="cuda")
         ptr = (self.ens_ws.data_ptr() + 255) // 256 * 256

@@ -128,8 +128,11 @@ sr_status validate_config(const sr_config* c) {
   if (c->n1 < 0 || c->n2 < 0 || c->n3 < 0 || c->n1 + c->n2 + c->n3 < 1)
     return fail(SR_ERR_INVALID_ARG, "block split needs n1, n2, n3 >= 0 and n1 + n2 + n3 >= 1");
   if (c->dtype != SR_F32 && c->dtype != SR_BF16) return fail(SR_ERR_INVALID_ARG, "bad dtype");
-  if (c->selector != SR_SEL_RANDOM && c->selector != SR_SEL_TOPK_L2)
+  if (c->selector != SR_SEL_RANDOM && c->selector != SR_SEL_TOPK_L2 &&
+      c->selector != SR_SEL_LAPLACIAN)
     return fail(SR_ERR_INVALID_ARG, "bad selector");
+  if (c->selector == SR_SEL_LAPLACIAN && (c->grid_w < 1 || c->L % c->grid_w != 0))
+    return fail(SR_ERR_INVALID_ARG, "the Laplacian selector needs grid_w >= 1 dividing L");
   if (c->shared_indices != 0 && c->shared_indices != 1)
     return fail(SR_ERR_INVALID_ARG, "shared_indices must be 0 or 1");
   if (!(c->ln_eps > 0.0f) || !std::isfinite(c->ln_eps))
@@ -165,8 +168,15 @@ struct sr_handle {
   std::vector<TraceRec> pending;
   std::vector<cudaEvent_t> pool;
   sr_trace_entry acc[SR_KERN_COUNT] = {};
+  // a batched view of a handle (the implicit ensemble's members as one batch)
+  // shares its owner's fault word and trace records
+  unsigned int* fault_ptr = nullptr;
+  sr_handle* owner = nullptr;
   void* at(size_t off) const { return ws + off; }
-  unsigned int* fault() const { return static_cast<unsigned int*>(at(plan.fault)); }
+  unsigned int* fault() const {
+    return fault_ptr ? fault_ptr : static_cast<unsigned int*>(at(plan.fault));
+  }
+  sr_handle* trace_owner() { return owner ? owner : this; }
   ~sr_handle() {
     for (auto& r : pending) { cudaEventDestroy(r.ev0); cudaEventDestroy(r.ev1); }
     for (auto e : pool) cudaEventDestroy(e);
@@ -194,7 +204,7 @@ struct TraceScope {
   TraceRec rec{};
   bool on = false;
   TraceScope(const sr_handle* hc, int kind, double flops, double bytes, cudaStream_t st)
-      : h(const_cast<sr_handle*>(hc)), s(st) {
+      : h(const_cast<sr_handle*>(hc)->trace_owner()), s(st) {
     if (!h->trace) return;
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
     if (cudaStreamIsCapturing(s, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return;
@@ -311,16 +321,21 @@ sr_status do_select(sr_handle* h, const float* x, int32_t K, uint64_t seed, int3
                     cudaStream_t s, bool score_ready = false) {
   const sr_config& c = h->cfg;
   const bool norms = c.selector == SR_SEL_TOPK_L2 && !score_ready;
+  const bool lap = c.selector == SR_SEL_LAPLACIAN;
+  // the Laplacian reads every token once (its four neighbours come from L2)
   const double sel_bytes = 4.0 * c.B * K +
-      (c.selector == SR_SEL_TOPK_L2 ? 4.0 * c.B * c.L : 0.0) +
-      (norms ? double(c.B) * c.L * c.D * 4.0 : 0.0);
+      (c.selector != SR_SEL_RANDOM ? 4.0 * c.B * c.L : 0.0) +
+      (norms || lap ? double(c.B) * c.L * c.D * 4.0 : 0.0);
   TraceScope t(h, SR_KERN_SELECT, 0.0, sel_bytes, s);
   if (c.selector == SR_SEL_RANDOM) {
     SR_CUDA(sr::launch_select_random(c.B, c.L, K, seed, c.shared_indices, idx, s), "select_random");
   } else {
     float* score = static_cast<float*>(h->at(h->plan.score));
     if (norms) SR_CUDA(sr::launch_token_sq_norms(h->dt, x, c.B * c.L, c.D, score, s), "token norms");
-    const int parts = norms ? 1 : sr::gemm_tc_sqnorm_parts(c.D);
+    if (lap)
+      SR_CUDA(sr::launch_token_laplacian(h->dt, x, c.B, c.L, c.grid_w, c.D, score, s),
+              "token Laplacian scores");
+    const int parts = norms || lap ? 1 : sr::gemm_tc_sqnorm_parts(c.D);
     SR_CUDA(sr::launch_select_topk(c.B, c.L, K, score, idx, s, parts), "select_topk");
   }
   return SR_OK;
@@ -382,13 +397,13 @@ sr_status sr_select(sr_handle* h, const void* x, float keep_ratio, uint64_t seed
   if (K < 0) return fail(SR_ERR_INVALID_ARG, "keep_ratio must lie in (0, 1]");
   if (K < 1) return fail(SR_ERR_INVALID_ARG, "K = floor(L * keep_ratio) is 0");
   if (!idx || !aligned(idx, 4)) return fail(SR_ERR_INVALID_ARG, "idx is NULL or misaligned");
-  if (h->cfg.selector == SR_SEL_TOPK_L2 && (!x || !aligned(x, 16)))
-    return fail(SR_ERR_INVALID_ARG, "top-K selection needs a 16-byte aligned x");
+  if (h->cfg.selector != SR_SEL_RANDOM && (!x || !aligned(x, 16)))
+    return fail(SR_ERR_INVALID_ARG, "score-based selection needs a 16-byte aligned x");
   if (K_out) *K_out = K;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   float* xs = nullptr;
-  if (h->cfg.selector == SR_SEL_TOPK_L2) {
-    // the norms are taken of the stored activations: widen them into the stream buffer
+  if (h->cfg.selector != SR_SEL_RANDOM) {
+    // the scores are taken of the stored activations: widen them into the stream buffer
     xs = static_cast<float*>(h->at(h->plan.xs));
     SR_CUDA(sr::launch_widen(h->dt, x, xs, size_t(h->cfg.B) * h->cfg.L * h->cfg.D, s), "widen x");
   }
@@ -451,20 +466,16 @@ sr_status widen_and_early(sr_handle* h, const void* x, const sr_block_weights* w
   return SR_OK;
 }
 
-// Everything after the dense-early blocks, in place on the fp32 stream xs:
-// selection, gather, the sparse middle with the delta scatter fused into its
-// last block, and the dense-late blocks (Alg. 1 after its dense-early loop).
-sr_status route_and_late(sr_handle* h, float* xs, const sr_block_weights* w, float keep_ratio,
-                         int32_t K, uint64_t seed, int32_t* idx_out, cudaStream_t s) {
+// The sparse middle (gather fused into its first LN1, delta scatter into its
+// last FC2) and the dense-late blocks, in place on the fp32 stream xs of h,
+// given the index set idx [B, K] (Alg. 1 after the selection).  With route false
+// the middle blocks run densely (r = 1, or no sparse blocks).
+sr_status blocks_after_select(sr_handle* h, float* xs, const sr_block_weights* w, bool route,
+                              int32_t K, const int32_t* idx, cudaStream_t s) {
   const sr_config& c = h->cfg;
   const int N = c.n1 + c.n2 + c.n3;
-  const bool route = keep_ratio < 1.0f && c.n2 > 0;
   sr_status st;
-  int32_t* idx = idx_out ? idx_out : static_cast<int32_t*>(h->at(h->plan.idx));
-  if (route || idx_out)
-    if ((st = do_select(h, xs, K, seed, idx, s, scores_fused(h))) != SR_OK) return st;
   if (route) {
-    // the gather of Eq. 8 is fused into the first sparse block's LN1
     float* hs = static_cast<float*>(h->at(h->plan.hs));
     for (int i = c.n1; i < c.n1 + c.n2; ++i) {
       const bool last = i == c.n1 + c.n2 - 1;
@@ -479,6 +490,28 @@ sr_status route_and_late(sr_handle* h, float* xs, const sr_block_weights* w, flo
   for (int i = c.n1 + c.n2; i < N; ++i)
     if ((st = run_block(h, xs, c.B, c.L, w[i], false, nullptr, nullptr, 0, s)) != SR_OK) return st;
   return SR_OK;
+}
+
+// Everything after the dense-early blocks, in place on the fp32 stream xs:
+// selection, gather, the sparse middle with the delta scatter fused into its
+// last block, and the dense-late blocks (Alg. 1 after its dense-early loop).
+sr_status route_and_late(sr_handle* h, float* xs, const sr_block_weights* w, float keep_ratio,
+                         int32_t K, uint64_t seed, int32_t* idx_out, cudaStream_t s) {
+  const sr_config& c = h->cfg;
+  const bool route = keep_ratio < 1.0f && c.n2 > 0;
+  sr_status st;
+  int32_t* idx = idx_out ? idx_out : static_cast<int32_t*>(h->at(h->plan.idx));
+  if (route || idx_out)
+    if ((st = do_select(h, xs, K, seed, idx, s, scores_fused(h))) != SR_OK) return st;
+  return blocks_after_select(h, xs, w, route, K, idx, s);
+}
+
+// The config of M members of the implicit ensemble run as one batch of M * B
+// samples (member m's sample b is sample m * B + b).
+sr_config ensemble_batch_config(const sr_config& c, int32_t M) {
+  sr_config e = c;
+  e.B = c.B * M;
+  return e;
 }
 
 }  // namespace
@@ -505,10 +538,14 @@ sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, flo
   return SR_OK;
 }
 
-size_t sr_ensemble_workspace_bytes(const sr_config* cfg) {
-  if (validate_config(cfg) != SR_OK) return 0;
-  // the dense-early result and the fp32 sum of the members
-  return 2 * align_up(size_t(cfg->B) * cfg->L * cfg->D * sizeof(float));
+size_t sr_ensemble_workspace_bytes(const sr_config* cfg, int32_t M, float max_keep_ratio) {
+  if (validate_config(cfg) != SR_OK || M < 1) return 0;
+  if (double(cfg->B) * M > 2147483647.0) return 0;
+  const int32_t K = keep_count(cfg->L, max_keep_ratio);
+  if (K < 0) return 0;
+  const sr_config e = ensemble_batch_config(*cfg, M);
+  if (validate_config(&e) != SR_OK) return 0;
+  return make_plan(e, K).total;
 }
 
 sr_status sr_forward_ensemble(sr_handle* h, const void* x, const sr_block_weights* w,
@@ -521,8 +558,11 @@ sr_status sr_forward_ensemble(sr_handle* h, const void* x, const sr_block_weight
   if (M < 1 || !seeds) return fail(SR_ERR_INVALID_ARG, "need M >= 1 seeds");
   const sr_config& c = h->cfg;
   const size_t n = size_t(c.B) * c.L * c.D;
-  const size_t fbytes = align_up(n * sizeof(float));
-  if (!ens_workspace || !aligned(ens_workspace, kAlign) || ens_ws_bytes < 2 * fbytes)
+  if (double(c.B) * M > 2147483647.0) return fail(SR_ERR_UNSUPPORTED, "B * M too large");
+  const sr_config ec = ensemble_batch_config(c, M);
+  if ((st = validate_config(&ec)) != SR_OK) return st;
+  const Plan ep = make_plan(ec, K > 0 ? K : 0);
+  if (!ens_workspace || !aligned(ens_workspace, kAlign) || ens_ws_bytes < ep.total)
     return fail(SR_ERR_WORKSPACE, "ensemble workspace NULL, misaligned or too small");
   if (members_out && !aligned(members_out, 16))
     return fail(SR_ERR_INVALID_ARG, "members_out must be 16-byte aligned");
@@ -540,37 +580,58 @@ sr_status sr_forward_ensemble(sr_handle* h, const void* x, const sr_block_weight
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   float* xs = static_cast<float*>(h->at(h->plan.xs));
-  float* xe = static_cast<float*>(ens_workspace);
-  float* acc = reinterpret_cast<float*>(static_cast<char*>(ens_workspace) + fbytes);
   const sr::PdlScope pdl(false);
   // the dense-early blocks do not depend on the seed: once for all members
   if ((st = widen_and_early(h, x, w, xs, s)) != SR_OK) return st;
   const sr::PdlScope pdl_rest(!h->trace);
-  if (M > 1) {
-    TraceScope t(h, SR_KERN_COPY, 0.0, 8.0 * n, s);
-    SR_CUDA(sr::launch_accumulate(xs, xe, n, true, s), "keep the dense-early result");
-  }
-  for (int32_t m = 0; m < M; ++m) {
-    if (m > 0) {
-      TraceScope t(h, SR_KERN_COPY, 0.0, 8.0 * n, s);
-      SR_CUDA(sr::launch_accumulate(xe, xs, n, true, s), "restore the dense-early result");
-    }
-    int32_t* idx_m = idx_out ? idx_out + size_t(m) * c.B * K : nullptr;
-    if ((st = route_and_late(h, xs, w, keep_ratio, K, seeds[m], idx_m, s)) != SR_OK) return st;
-    if (members_out) {
-      TraceScope t(h, SR_KERN_COPY, 0.0, double(n) * (h->es + 4.0), s);
+  const bool route = keep_ratio < 1.0f && c.n2 > 0;
+  if (!route) {
+    // nothing is routed: every member is the same dense forward, and so is
+    // their mean
+    for (int32_t m = 0; idx_out && m < M; ++m)
+      if ((st = do_select(h, xs, K, seeds[m], idx_out + size_t(m) * c.B * K, s, scores_fused(h))) !=
+          SR_OK)
+        return st;
+    if ((st = blocks_after_select(h, xs, w, false, K, nullptr, s)) != SR_OK) return st;
+    TraceScope t(h, SR_KERN_COPY, 0.0, double(n) * (h->es + 4.0) * (1 + (members_out ? M : 0)), s);
+    for (int32_t m = 0; members_out && m < M; ++m)
       SR_CUDA(sr::launch_narrow(h->dt, xs, static_cast<char*>(members_out) + size_t(m) * bytes, n, s),
               "narrow member");
-    }
-    if (M > 1) {
-      TraceScope t(h, SR_KERN_COPY, 0.0, (m == 0 ? 8.0 : 12.0) * n, s);
-      SR_CUDA(sr::launch_accumulate(xs, acc, n, m == 0, s), "sum of the members");
-    }
+    SR_CUDA(sr::launch_narrow(h->dt, xs, out, n, s), "narrow out");
+    return SR_OK;
+  }
+  // the M members run as one batch of M * B samples on a view of the handle
+  // over the ensemble workspace; each member's index set is selected from the
+  // shared dense-early result with its own seed, exactly as sr_forward does
+  sr_handle v;
+  v.cfg = ec;
+  v.dt = h->dt;
+  v.es = h->es;
+  v.ws = static_cast<char*>(ens_workspace);
+  v.ws_bytes = ens_ws_bytes;
+  v.Kmax = K;
+  v.plan = ep;
+  v.trace = h->trace;
+  v.fault_ptr = h->fault();
+  v.owner = h;
+  float* xe = static_cast<float*>(v.at(ep.xs));
+  int32_t* idx = idx_out ? idx_out : static_cast<int32_t*>(v.at(ep.idx));
+  for (int32_t m = 0; m < M; ++m)
+    if ((st = do_select(h, xs, K, seeds[m], idx + size_t(m) * c.B * K, s, scores_fused(h))) != SR_OK)
+      return st;
+  {
+    TraceScope t(h, SR_KERN_COPY, 0.0, 4.0 * double(n) * (1 + M), s);
+    SR_CUDA(sr::launch_replicate(xs, xe, n, M, s), "replicate the dense-early result");
+  }
+  if ((st = blocks_after_select(&v, xe, w, true, K, idx, s)) != SR_OK) return st;
+  if (members_out) {
+    TraceScope t(h, SR_KERN_COPY, 0.0, double(M) * n * (h->es + 4.0), s);
+    SR_CUDA(sr::launch_narrow(h->dt, xe, members_out, size_t(M) * n, s), "narrow members");
   }
   {
-    // the mean of the members' fp32 results, rounded once
-    TraceScope t(h, SR_KERN_COPY, 0.0, double(n) * (h->es + 4.0), s);
-    SR_CUDA(sr::launch_narrow(h->dt, M > 1 ? acc : xs, out, n, s, 1.0f / float(M)), "narrow mean");
+    // the mean of the members' fp32 results (summed in member order), rounded once
+    TraceScope t(h, SR_KERN_COPY, 0.0, double(n) * (4.0 * M + h->es), s);
+    SR_CUDA(sr::launch_mean_narrow(h->dt, xe, M, n, 1.0f / float(M), out, s), "narrow mean");
   }
   return SR_OK;
 }

@@ -60,6 +60,12 @@ cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared,
 // stores), its square accumulated in fp32.
 cudaError_t launch_token_sq_norms(DType dt, const float* x, int rows, int D, float* score,
                                   cudaStream_t s);
+// Laplacian score of every token of the fp32 stream x [B*L, D] into score [B*L]:
+// tokens row-major on a patch grid grid_w wide, 5-point stencil with periodic
+// longitude and the first and last rows reflected; each value rounded to the
+// storage dtype dt, the squared norm of the stencil accumulated in fp32.
+cudaError_t launch_token_laplacian(DType dt, const float* x, int B, int L, int grid_w, int D,
+                                   float* score, cudaStream_t s);
 // K largest scores per sample (ties to the lower index), sorted indices.  A
 // token's score is the sum of `parts` consecutive partial sums (score
 // [B*L][parts]), added in order.
@@ -75,8 +81,12 @@ cudaError_t launch_widen(DType dt, const void* x, float* y, size_t n, cudaStream
 // narrow rounds scale * x once to the storage dtype
 cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStream_t s,
                           float scale = 1.0f);
-// acc = x (first) or acc += x, fp32, n % 4 == 0
-cudaError_t launch_accumulate(const float* x, float* acc, size_t n, bool first, cudaStream_t s);
+// y[m * n + i] = x[i] for m < M, fp32, n % 4 == 0
+cudaError_t launch_replicate(const float* x, float* y, size_t n, int M, cudaStream_t s);
+// y = scale * sum_m x[m * n + i] rounded once to the storage dtype, the sum in
+// fp32 in member order, n % 8 == 0
+cudaError_t launch_mean_narrow(DType dt, const float* x, int M, size_t n, float scale, void* y,
+                               cudaStream_t s);
 
 // ---- LayerNorm over D from the fp32 stream into the storage dtype ---------
 //      y = (x - mean) / sqrt(var + eps) * g + b

@@ -1,9 +1,10 @@
 // Row-wise HBM-bound kernels on the fp32 residual stream: LayerNorm (the LN of
 // the pre-LN block, Sec. 3.3 Eq. 11), which for the first sparse block also
 // performs the routed-token gather (Eq. 8) through the index set; the
-// conversions between the caller's storage dtype and the stream; and the fp32
-// sum of an implicit ensemble's members.  One warp owns one row; rows move as
-// 16-byte vectors, all loads of a row are issued before any use.
+// conversions between the caller's storage dtype and the stream; and the
+// implicit ensemble's copies of the dense-early result and mean of its members.
+// In LayerNorm one warp owns one row; rows move as 16-byte vectors, all loads
+// of a row are issued before any use.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -103,21 +104,49 @@ widen_kernel(const T* __restrict__ x, float* __restrict__ y, size_t nvec, float*
   }
 }
 
-// acc = x (first) or acc += x over the fp32 stream, 4-float vectors
+// y[m] = x for m = 0 .. M-1 (the implicit ensemble's members start from the
+// same dense-early result), 4-float vectors
 __global__ void __launch_bounds__(256)
-accumulate_kernel(const float* __restrict__ x, float* __restrict__ acc, size_t nvec, int first) {
+replicate_kernel(const float* __restrict__ x, float* __restrict__ y, size_t nvec, int M) {
   pdl_wait();      // the previous kernel's writes are visible from here
   pdl_trigger();
   const float4* xv = reinterpret_cast<const float4*>(x);
-  float4* av = reinterpret_cast<float4*>(acc);
+  float4* yv = reinterpret_cast<float4*>(y);
   for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
        i += size_t(gridDim.x) * blockDim.x) {
-    float4 v = __ldg(xv + i);
-    if (!first) {
-      const float4 a = av[i];
-      v = make_float4(a.x + v.x, a.y + v.y, a.z + v.z, a.w + v.w);
+    const float4 v = __ldg(xv + i);
+    for (int m = 0; m < M; ++m) yv[size_t(m) * nvec + i] = v;
+  }
+}
+
+// y = scale * (x[0] + x[1] + ... + x[M-1]) rounded once to the storage dtype T,
+// the sum in fp32 in member order (x: M consecutive fp32 streams of nvec vectors)
+template <typename T>
+__global__ void __launch_bounds__(256)
+mean_narrow_kernel(const float* __restrict__ x, int M, size_t nvec, float scale, T* __restrict__ y) {
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
+  constexpr int V = Elem<T>::kVec;
+  const size_t n4 = nvec * (V / 4);            // float4 vectors per member
+  for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
+       i += size_t(gridDim.x) * blockDim.x) {
+    float f[V];
+    const float4* in = reinterpret_cast<const float4*>(x) + i * (V / 4);
+#pragma unroll
+    for (int q = 0; q < V / 4; ++q) {
+      const float4 v4 = __ldg(in + q);
+      f[4 * q] = v4.x; f[4 * q + 1] = v4.y; f[4 * q + 2] = v4.z; f[4 * q + 3] = v4.w;
     }
-    av[i] = v;
+    for (int m = 1; m < M; ++m) {
+#pragma unroll
+      for (int q = 0; q < V / 4; ++q) {
+        const float4 v4 = __ldg(in + size_t(m) * n4 + q);
+        f[4 * q] += v4.x; f[4 * q + 1] += v4.y; f[4 * q + 2] += v4.z; f[4 * q + 3] += v4.w;
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < V; ++e) f[e] *= scale;
+    reinterpret_cast<uint4*>(y)[i] = pack16(f);
   }
 }
 
@@ -183,10 +212,21 @@ cudaError_t launch_narrow(DType dt, const float* x, void* y, size_t n, cudaStrea
                   static_cast<float*>(y), nvec, scale);
 }
 
-cudaError_t launch_accumulate(const float* x, float* acc, size_t n, bool first, cudaStream_t s) {
+cudaError_t launch_replicate(const float* x, float* y, size_t n, int M, cudaStream_t s) {
   const size_t nvec = n / 4;
-  return launch_k(accumulate_kernel, dim3(grid_for(nvec)), dim3(256), 0, s, 1, x, acc, nvec,
-                  first ? 1 : 0);
+  return launch_k(replicate_kernel, dim3(grid_for(nvec)), dim3(256), 0, s, 1, x, y, nvec, M);
+}
+
+cudaError_t launch_mean_narrow(DType dt, const float* x, int M, size_t n, float scale, void* y,
+                               cudaStream_t s) {
+  if (dt == DType::BF16) {
+    const size_t nvec = n / 8;
+    return launch_k(mean_narrow_kernel<bf16>, dim3(grid_for(nvec)), dim3(256), 0, s, 1, x, M, nvec,
+                    scale, static_cast<bf16*>(y));
+  }
+  const size_t nvec = n / 4;
+  return launch_k(mean_narrow_kernel<float>, dim3(grid_for(nvec)), dim3(256), 0, s, 1, x, M, nvec,
+                  scale, static_cast<float*>(y));
 }
 
 cudaError_t launch_layernorm(DType dt, const float* x, const void* g, const void* b, void* y,

@@ -1,14 +1,16 @@
-// Token selection (Sec. 3.2 random selection; App. B.2 activation-norm selector).
+// Token selection (Sec. 3.2 random selection; App. B.2 activation-norm and
+// gradient (Laplacian) selectors).
 //
-// Both selectors reduce to one primitive: per sample, keep the K smallest keys
+// All selectors reduce to one primitive: per sample, keep the K smallest keys
 // (ties broken by the lower token index) and emit their token indices in
 // ascending order.  One CTA owns one sample: its L keys sit in shared memory, a
 // most-significant-digit radix select (8-bit digits) finds the K-th smallest key
 // T and how many keys equal to T must be kept, and an ordered block-wide
 // compaction writes the selected indices, which come out sorted by
 // construction.  Work per sample is O(L * passes); HBM traffic is the index
-// write (4 B per selected token) plus, for the top-K selector, the scores: one
-// pass over x computes them, unless the forward's FC2 epilogue already has.
+// write (4 B per selected token) plus, for the score-based selectors, the
+// scores: one pass over x computes them (the L2 norms, or the Laplacian on the
+// patch grid), unless the forward's FC2 epilogue already has the norms.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -192,9 +194,62 @@ token_sq_norms_kernel(const float* __restrict__ x, int rows, int D, float* __res
   if (lane == 0) score[warp] = acc;
 }
 
+// One warp per token (i, j) of the patch grid: the 5-point Laplacian of its row
+// of the stream, x(i-1,j) + x(i+1,j) + x(i,j-1) + x(i,j+1) - 4 x(i,j), with
+// longitude periodic and the first and last latitude rows reflected onto
+// themselves; every value rounded to the storage dtype T first, the squared
+// norm of the stencil accumulated in fp32.  Each row is read by five warps, so
+// the neighbours' reads come from L2.
+template <typename T>
+__global__ void __launch_bounds__(256)
+token_laplacian_kernel(const float* __restrict__ x, int B, int L, int W, int D,
+                       float* __restrict__ score) {
+  pdl_wait();      // the previous kernel's writes are visible from here
+  pdl_trigger();
+  const int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (t >= B * L) return;
+  const int b = t / L, tok = t % L;
+  const int H = L / W, i = tok / W, j = tok % W;
+  const size_t base = size_t(b) * L;
+  const float4* c = reinterpret_cast<const float4*>(x + (base + tok) * D);
+  const float4* n = reinterpret_cast<const float4*>(x + (base + size_t(i > 0 ? i - 1 : 0) * W + j) * D);
+  const float4* so = reinterpret_cast<const float4*>(
+      x + (base + size_t(i + 1 < H ? i + 1 : H - 1) * W + j) * D);
+  const float4* w = reinterpret_cast<const float4*>(x + (base + size_t(i) * W + (j + W - 1) % W) * D);
+  const float4* e = reinterpret_cast<const float4*>(x + (base + size_t(i) * W + (j + 1) % W) * D);
+  auto rd = [](float v) { return Elem<T>::to_f(Elem<T>::from_f(v)); };
+  float acc = 0.f;
+  for (int v = lane; v < D / 4; v += 32) {
+    const float4 qc = __ldg(c + v), qn = __ldg(n + v), qs = __ldg(so + v), qw = __ldg(w + v),
+                 qe = __ldg(e + v);
+    const float fc[4] = {qc.x, qc.y, qc.z, qc.w}, fn[4] = {qn.x, qn.y, qn.z, qn.w},
+                fs[4] = {qs.x, qs.y, qs.z, qs.w}, fw[4] = {qw.x, qw.y, qw.z, qw.w},
+                fe[4] = {qe.x, qe.y, qe.z, qe.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float lap = ((rd(fn[k]) + rd(fs[k])) + (rd(fw[k]) + rd(fe[k]))) - 4.0f * rd(fc[k]);
+      acc = fmaf(lap, lap, acc);
+    }
+  }
+  acc = warp_sum(acc);
+  if (lane == 0) score[t] = acc;
+}
+
 }  // namespace
 
 int select_max_L() { return kSelMaxL; }
+
+cudaError_t launch_token_laplacian(DType dt, const float* x, int B, int L, int grid_w, int D,
+                                   float* score, cudaStream_t s) {
+  if (grid_w < 1 || L % grid_w != 0 || D % 4 != 0) return cudaErrorInvalidValue;
+  const int blocks = (B * L + 7) / 8;
+  if (dt == DType::BF16)
+    return launch_k(token_laplacian_kernel<bf16>, dim3(blocks), dim3(256), 0, s, 1, x, B, L, grid_w,
+                    D, score);
+  return launch_k(token_laplacian_kernel<float>, dim3(blocks), dim3(256), 0, s, 1, x, B, L, grid_w, D,
+                  score);
+}
 
 cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared, int32_t* idx,
                                  cudaStream_t s) {

@@ -45,13 +45,18 @@ class Workload:
     n3: int
     keep_ratio: float
     dtype: str           # "f32" or "bf16"
-    selector: str = "random"   # "random" or "topk_l2"
+    selector: str = "random"   # "random", "topk_l2" or "laplacian"
     crop_last_row: bool = False  # generate grid_h + 1 latitudes, drop the last
     seed_index: int = 0
 
     @property
     def L(self) -> int:
         return (self.grid_h // self.patch) * (self.grid_w // self.patch)
+
+    @property
+    def grid_wp(self) -> int:
+        """Tokens per latitude row of the patch grid."""
+        return self.grid_w // self.patch
 
     @property
     def N(self) -> int:
@@ -97,7 +102,7 @@ WORKLOADS: Dict[str, Workload] = {
 }
 
 SWEEP_RATIOS = (1.0, 0.5, 0.25, 0.125)
-SWEEP_SELECTORS = ("random", "topk_l2")
+SWEEP_SELECTORS = ("random", "topk_l2", "laplacian")
 
 
 def sweep_workloads() -> List[Workload]:

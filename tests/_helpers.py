@@ -73,7 +73,7 @@ def gpu_forward(wl, x, weights, keep_ratio=None, seed=None, selector=None, share
     n1, n2, n3 = n_split or (wl.n1, wl.n2, wl.n3)
     r = wl.keep_ratio if keep_ratio is None else keep_ratio
     cfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, n1, n2, n3, dtype=wl.dtype,
-                        selector=selector or wl.selector, shared=shared)
+                        selector=selector or wl.selector, shared=shared, grid_w=wl.grid_wp)
     enc = b.Encoder(cfg, max_keep_ratio=r)
     xd, wd = to_device(x, weights[:n1 + n2 + n3])
     warr = b.weights_array(wd)

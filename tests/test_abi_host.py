@@ -36,10 +36,13 @@ def test_invalid_configs_rejected(L):
     from paper_2607_02829_gb300 import binding as b
     good = b.make_config(2, 512, 256, 4, 2, 2, 2, dtype="f32")
     assert b.sr_workspace_bytes(good, 0.25) > 0
+    lap = b.make_config(2, 512, 256, 4, 2, 2, 2, dtype="f32", selector="laplacian", grid_w=32)
+    assert b.sr_workspace_bytes(lap, 0.25) > 0
     bad = [
         dict(D=250), dict(heads=3), dict(B=0), dict(L=0), dict(n1=-1),
         dict(n1=0, n2=0, n3=0), dict(dtype=7), dict(selector=5), dict(shared_indices=2),
         dict(ln_eps=0.0), dict(mlp_hidden=100), dict(L=100000),
+        dict(selector=2), dict(selector=2, grid_w=7), dict(selector=2, grid_w=-64),
     ]
     for kw in bad:
         c = b.make_config(2, 512, 256, 4, 2, 2, 2, dtype="f32")
@@ -129,10 +132,16 @@ def test_routed_only_workspace_is_smaller_and_rejects_the_dense_path(L):
 def test_ensemble_workspace_and_argument_errors(L):
     from paper_2607_02829_gb300 import binding as b
     cfg = b.make_config(2, 512, 256, 4, 1, 2, 1, dtype="f32")
-    ens = b.sr_ensemble_workspace_bytes(cfg)
+    ens = b.sr_ensemble_workspace_bytes(cfg, 2, 0.25)
+    # the batch of M * B samples: at least its fp32 stream
     assert ens >= 2 * 2 * 512 * 256 * 4
+    assert b.sr_ensemble_workspace_bytes(cfg, 3, 0.25) > ens
     bad = b.make_config(2, 512, 250, 4, 1, 2, 1, dtype="f32")
-    assert b.sr_ensemble_workspace_bytes(bad) == 0
+    assert b.sr_ensemble_workspace_bytes(bad, 2, 0.25) == 0
+    assert b.sr_ensemble_workspace_bytes(cfg, 0, 0.25) == 0
+    assert b.sr_ensemble_workspace_bytes(cfg, 2, 1.5) == 0
+    big = b.make_config(64, 16200, 1024, 16, 4, 16, 4, dtype="bf16")
+    assert b.sr_ensemble_workspace_bytes(big, 8, 0.25) == 0      # 2^31-element limit
     h = _handle(b, cfg, b.sr_workspace_bytes(cfg, 0.25))
     try:
         w = (b.sr_block_weights * 4)()

@@ -5,10 +5,12 @@
   tests/golden/ (written by tests/golden/make_c4_golden.py, which calls only
   the oracle) as a quick check, then the whole oracle forward element by
   element; the bit-exact index set and unselected-row passthrough.
-* keep-ratio x selector sweep on the 1.40625 deg model: index sets for every
-  point, r = 1 bitwise equal to the dense stack, and the whole output of every
-  point against the oracle (r = 1 against the oracle's dense stack; top-K
-  points given the GPU's index set, which the index test checks separately).
+* keep-ratio x selector sweep on the 1.40625 deg model (random, top-K L2 norm,
+  and the Laplacian selector): index sets for every point, r = 1 bitwise equal
+  to the dense stack, and the whole output against the oracle at every point of
+  the random and top-K selectors and at r = 0.25 of the Laplacian one (r = 1
+  against the oracle's dense stack; score-based points given the GPU's index
+  set, which the index test checks separately).
   The oracle's dense-early stage does not depend on r or the selector, so it
   runs once for the sweep.
 
@@ -92,7 +94,7 @@ def sweep_inputs():
     return synth.make_inputs(wl)
 
 
-@pytest.mark.parametrize("selector", ["random", "topk_l2"])
+@pytest.mark.parametrize("selector", ["random", "topk_l2", "laplacian"])
 @pytest.mark.parametrize("r", [1.0, 0.5, 0.25, 0.125])
 def test_sweep_index_sets_and_passthrough(sweep_inputs, selector, r):
     wl = [w for w in synth.sweep_workloads() if w.selector == selector and w.keep_ratio == r][0]
@@ -112,8 +114,11 @@ def test_sweep_index_sets_and_passthrough(sweep_inputs, selector, r):
         # the GPU ranks the stored (bf16) block-n1 output; the oracle ranks the same
         # values in fp64: equal sets, or differences only inside the fp32 tie band
         x0 = synth.stored_as_f64(pre)
-        s = o.token_sq_norms(x0)
-        exp = o.select_topk_l2(x0, K)
+        if selector == "topk_l2":
+            s, exp = o.token_sq_norms(x0), o.select_topk_l2(x0, K)
+        else:
+            s = o.token_laplacian_scores(x0, wl.grid_wp)
+            exp = o.select_topk_laplacian(x0, K, wl.grid_wp)
         for b in range(wl.B):
             diff = set(idx[b].tolist()) ^ set(exp[b].tolist())
             kth = np.sort(s[b])[::-1][K - 1]
@@ -130,7 +135,7 @@ def sweep_oracle_early(sweep_inputs):
 
 
 @pytest.mark.parametrize("selector,r", [("random", 1.0), ("random", 0.5), ("topk_l2", 0.5),
-                                        ("random", 0.25), ("topk_l2", 0.25),
+                                        ("random", 0.25), ("topk_l2", 0.25), ("laplacian", 0.25),
                                         ("random", 0.125), ("topk_l2", 0.125)])
 def test_sweep_forward_matches_oracle(sweep_inputs, sweep_oracle_early, selector, r):
     wl = [w for w in synth.sweep_workloads() if w.selector == selector and w.keep_ratio == r][0]
@@ -144,7 +149,7 @@ def test_sweep_forward_matches_oracle(sweep_inputs, sweep_oracle_early, selector
             assert np.array_equal(idx, o.select_random(wl.B, wl.L, o.keep_count(wl.L, r),
                                                        wl.select_seed))
         # the routed and dense-late stages of Alg. 1 on the oracle's dense-early
-        # output; the random index set is drawn again by the oracle, the top-K
+        # output; the random index set is drawn again by the oracle, a score-based
         # set is the GPU's (equal to the oracle's up to the fp32 tie band)
         ref, _ = o.forward(x_early, wf[wl.n1:], 0, wl.n2, wl.n3, wl.heads, r,
                            seed=wl.select_seed, idx=None if selector == "random" else idx,

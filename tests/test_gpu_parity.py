@@ -30,7 +30,7 @@ def _oracle(wl, x, ws, keep_ratio=None, seed=None, selector=None, n_split=None, 
     return o.forward(xf, wf, n1, n2, n3, wl.heads,
                      wl.keep_ratio if keep_ratio is None else keep_ratio,
                      seed=wl.select_seed if seed is None else seed,
-                     selector=selector or wl.selector, idx=idx, threads=8)
+                     selector=selector or wl.selector, idx=idx, threads=8, grid_w=wl.grid_wp)
 
 
 def _tiny(dtype, B=2, L=200, heads=2, split=(1, 2, 1), r=0.25, selector="random"):
@@ -198,6 +198,45 @@ def test_forward_parity_topk_selector_small(dtype, heads):
     assert np.array_equal(idx, o.select_topk_l2(synth.stored_as_f64(x0), 64))
     again, idx2 = gpu_forward(wl, x, ws)
     assert torch.equal(out, again) and np.array_equal(idx, idx2)     # reproducible
+
+
+# the Laplacian selector on a 2-D patch grid (8 x 24 tokens): the index set
+# against the oracle's on the GPU's own pre-routing state, then the forward
+# against the oracle given the GPU's indices
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_forward_parity_laplacian_selector_small(dtype):
+    wl = synth.Workload(f"lap_{dtype}", B=2, grid_h=8, grid_w=24, channels=3, patch=1, D=128,
+                        heads=2, n1=2, n2=2, n3=1, keep_ratio=0.25, dtype=dtype,
+                        selector="laplacian", seed_index=78)
+    x, ws = synth.make_inputs(wl)
+    out, idx = gpu_forward(wl, x, ws)
+    x0, _ = gpu_forward(wl, x, ws, n_split=(2, 0, 0), want_idx=False)
+    xf = synth.stored_as_f64(x0)
+    K = o.keep_count(wl.L, wl.keep_ratio)
+    s = o.token_laplacian_scores(xf, wl.grid_wp)
+    exp = o.select_topk_laplacian(xf, K, wl.grid_wp)
+    for bb in range(wl.B):
+        kth = np.sort(s[bb])[::-1][K - 1]
+        diff = set(idx[bb].tolist()) ^ set(exp[bb].tolist())
+        assert all(abs(s[bb, i] - kth) <= 1e-5 * kth for i in diff), sorted(diff)
+    ref, _ = _oracle(wl, x, ws, idx=idx)
+    check_parity(f"small Laplacian {dtype}", synth.stored_as_f64(out), ref, TOL[dtype])
+
+
+@pytest.mark.parametrize("B,H,W,D,K", [(2, 8, 24, 64, 48), (1, 90, 180, 1024, 4050),
+                                       (3, 5, 1, 64, 2), (1, 1, 7, 64, 3)])
+def test_select_laplacian_integer_fields_exact(B, H, W, D, K):
+    # small integer values: every score is an exact integer on both sides, so
+    # the sets must be equal, ties included
+    from paper_2607_02829_gb300 import binding as b
+    g = torch.Generator().manual_seed(B * H * W + D)
+    x = torch.randint(-3, 4, (B, H * W, D), generator=g).to(torch.bfloat16)
+    cfg = b.make_config(B, H * W, D, D // 64, 0, 1, 0, dtype="bf16", selector="laplacian",
+                        grid_w=W)
+    enc = b.Encoder(cfg, max_keep_ratio=1.0)
+    idx = enc.select(x.cuda(), K / (H * W), 0).cpu().numpy()
+    enc.close()
+    assert np.array_equal(idx, o.select_topk_laplacian(synth.stored_as_f64(x), K, W))
 
 
 # ------------------------------------------------------------ implicit ensemble
