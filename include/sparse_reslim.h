@@ -181,7 +181,7 @@ sr_status sr_forward_ensemble(sr_handle* h, const void* x, const sr_block_weight
                               void* ens_workspace, size_t ens_ws_bytes, void* out,
                               void* members_out, int32_t* idx_out, void* stream);
 
-/* Asymmetric attention (Sec. 3.5, "Integration with generative forecasting";
+/* Asymmetric attention (Sec. 3.4, "Integration with generative forecasting";
  * Alg. 2): queries from one token set, keys and values from another, within
  * each sample and per head: out = softmax(q k^T / 8) v.  In the EDM model's
  * sparse stage the K routed tokens attend over the full L-token conditioning

@@ -206,7 +206,7 @@ def attention(qkv: np.ndarray, heads: int, pool: Optional[ThreadPoolExecutor] = 
 
 def cross_attention(q: np.ndarray, kv: np.ndarray, heads: int,
                     pool: Optional[ThreadPoolExecutor] = None) -> np.ndarray:
-    """Asymmetric attention (Sec. 3.5, "Integration with generative
+    """Asymmetric attention (Sec. 3.4, "Integration with generative
     forecasting"; Alg. 2): queries from one token set, keys and values from
     another, within each sample.  q: [B, Tq, D]; kv: [B, Tkv, 2D] with columns
     [0, D) = k and [D, 2D) = v, head h owning columns [h dh, (h+1) dh) of each.

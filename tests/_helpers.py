@@ -40,20 +40,20 @@ def max_norm_rel(y, o):
 
 
 # (case, max-norm relative error, 99.9th percentile of |y - o| / max|o|, bar,
-# elements compared), in test order; the session summary prints them
+# elements compared, note), in test order; the session summary prints them
 PARITY_RECORDS = []
 
 
-def check_parity(case, y, o, tol):
+def check_parity(case, y, o, tol, note=""):
     """Asserts max|y - o| / max|o| <= tol and records that error together with
-    the elementwise 99.9th-percentile error |y - o| / max|o|."""
+    the elementwise 99.9th-percentile error |y - o| / max|o| (and a note)."""
     y = np.asarray(y, dtype=np.float64)
     o = np.asarray(o, dtype=np.float64)
     scale = max(float(np.abs(o).max()), 1e-300)
     e = np.abs(y - o).ravel() / scale
     err = float(e.max())
     p999 = float(np.quantile(e, 0.999))
-    PARITY_RECORDS.append((case, err, p999, tol, int(e.size)))
+    PARITY_RECORDS.append((case, err, p999, tol, int(e.size), note))
     assert err <= tol, f"{case}: max-norm relative error {err:.3e} exceeds {tol:.0e}"
     return err
 

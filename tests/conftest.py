@@ -28,11 +28,11 @@ def pytest_terminal_summary(terminalreporter):
     tr = terminalreporter
     tr.write_sep("-", "output parity against the fp64 oracle")
     tr.write_line(f"{'case':58s} {'max-norm':>10s} {'p99.9':>10s} {'bar':>7s} {'elements':>11s}")
-    for case, err, p999, tol, n in PARITY_RECORDS:
-        tr.write_line(f"{case:58s} {err:10.3e} {p999:10.3e} {tol:7.0e} {n:11d}")
+    for case, err, p999, tol, n, note in PARITY_RECORDS:
+        tr.write_line(f"{case:58s} {err:10.3e} {p999:10.3e} {tol:7.0e} {n:11d}  {note}")
     path = os.environ.get("SR_PARITY_REPORT")
     if path:
         import json
         with open(path, "w") as f:
-            json.dump([{"case": c, "max_norm_rel": e, "p999_rel": p, "bar": t, "elements": n}
-                       for c, e, p, t, n in PARITY_RECORDS], f, indent=1)
+            json.dump([{"case": c, "max_norm_rel": e, "p999_rel": p, "bar": t, "elements": n,
+                        "note": nt} for c, e, p, t, n, nt in PARITY_RECORDS], f, indent=1)

@@ -17,6 +17,7 @@
 Every output comparison records its max-norm and 99.9th-percentile errors.
 """
 import os
+import time
 
 import numpy as np
 import pytest
@@ -82,10 +83,14 @@ def test_c4_full_forward_matches_oracle():
     wl = synth.WORKLOADS["c4_0p25deg_bf16"]
     x, ws = synth.make_inputs(wl)
     out, idx = gpu_forward(wl, x, ws)
-    ref, ridx = o.forward(synth.stored_as_f64(x), o.as_f64_weights(ws), wl.n1, wl.n2, wl.n3,
-                          wl.heads, wl.keep_ratio, seed=wl.select_seed, threads=THREADS)
+    xf, wf = synth.stored_as_f64(x), o.as_f64_weights(ws)
+    t0 = time.perf_counter()
+    ref, ridx = o.forward(xf, wf, wl.n1, wl.n2, wl.n3, wl.heads, wl.keep_ratio,
+                          seed=wl.select_seed, threads=THREADS)
+    oracle_s = time.perf_counter() - t0
     assert np.array_equal(idx, ridx)
-    check_parity("c4_0p25deg_bf16 (full output)", synth.stored_as_f64(out), ref, TOL)
+    check_parity("c4_0p25deg_bf16 (full output)", synth.stored_as_f64(out), ref, TOL,
+                 note=f"oracle forward {oracle_s:.1f} s on {THREADS} threads")
 
 
 @pytest.fixture(scope="module")

@@ -414,7 +414,7 @@ def test_ensemble_passthrough_tokens():
 
 # ------------------------------------------------------------------ asymmetric attention
 def test_cross_attention_against_torch_sdpa_and_bruteforce():
-    # queries and keys/values of different lengths (Sec. 3.5: Q from the K routed
+    # queries and keys/values of different lengths (Sec. 3.4: Q from the K routed
     # tokens, K and V from the L-token conditioning sequence)
     rng = np.random.default_rng(5)
     B, Tq, Tkv, H, dh = 2, 7, 13, 3, 8
