@@ -4,10 +4,10 @@
 // All selectors reduce to one primitive: per sample, keep the K smallest keys
 // (ties broken by the lower token index) and emit their token indices in
 // ascending order.  One CTA owns one sample: its L keys sit in shared memory, a
-// most-significant-digit radix select (8-bit digits) finds the K-th smallest key
-// T and how many keys equal to T must be kept, and an ordered block-wide
-// compaction writes the selected indices, which come out sorted by
-// construction.  Work per sample is O(L * passes); HBM traffic is the index
+// most-significant-digit radix select (8-bit digits, stopping once the K-th
+// smallest key's digit bin is kept whole) finds the threshold and how many keys
+// equal to it must be kept, and an ordered block-wide compaction writes the
+// selected indices, which come out sorted by construction.  Work per sample is O(L * passes); HBM traffic is the index
 // write (4 B per selected token) plus, for the score-based selectors, the
 // scores: one pass over x computes them (the L2 norms, or the Laplacian on the
 // patch grid), unless the forward's FC2 epilogue already has the norms.
@@ -35,32 +35,43 @@ __device__ __forceinline__ uint32_t desc_key(float score) {
   return ~asc;
 }
 
-// Block-wide exclusive prefix count of `flag` in thread order; returns the
-// thread's exclusive prefix and writes the block total to *total.
-__device__ __forceinline__ int block_excl_count(bool flag, int* warp_tot, int* total) {
+// Block-wide exclusive prefix sum of `v` in thread order; returns the thread's
+// exclusive prefix and writes the block total to *total.
+__device__ __forceinline__ int block_excl_sum(int v, int* warp_tot, int* total) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const unsigned bal = __ballot_sync(0xffffffffu, flag);
-  const int in_warp = __popc(bal & ((1u << lane) - 1u));
-  if (lane == 0) warp_tot[warp] = __popc(bal);
+  int incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  if (lane == 31) warp_tot[warp] = incl;
   __syncthreads();
   if (warp == 0) {
     const int nw = blockDim.x >> 5;
-    int v = lane < nw ? warp_tot[lane] : 0;
-    int incl = v;
+    const int w = lane < nw ? warp_tot[lane] : 0;
+    int wi = w;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      int t = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += t;
+      const int t = __shfl_up_sync(0xffffffffu, wi, o);
+      if (lane >= o) wi += t;
     }
-    if (lane < nw) warp_tot[lane] = incl - v;   // exclusive warp offsets
-    if (lane == 31) *total = incl;
+    if (lane < nw) warp_tot[lane] = wi - w;      // exclusive warp offsets
+    if (lane == 31) *total = wi;
   }
   __syncthreads();
-  const int r = warp_tot[warp] + in_warp;
+  const int r = warp_tot[warp] + incl - v;
   __syncthreads();   // warp_tot is reused by the next call
   return r;
 }
 
+// Writes, in ascending order, the indices of the K smallest of the L keys
+// (ties to the lower index).  A most-significant-digit radix select (8-bit
+// digits) narrows a prefix of the K-th smallest key; it stops as soon as every
+// key under the current prefix is kept, which for random keys happens after a
+// few digits.  The compaction then gives each thread a contiguous range of
+// indices: two block scans (of the kept keys equal to the threshold, then of
+// all kept keys) place every index.
 template <typename Key>
 __device__ void select_smallest_sorted(const Key* keys, int L, int K, int32_t* out_idx) {
   __shared__ int hist[256];
@@ -68,8 +79,9 @@ __device__ void select_smallest_sorted(const Key* keys, int L, int K, int32_t* o
   __shared__ int s_total;
   __shared__ Key s_prefix;
   __shared__ int s_krem;
+  __shared__ int s_whole;      // every key under the prefix is kept
   const int tid = threadIdx.x;
-  if (tid == 0) { s_prefix = 0; s_krem = K; }
+  if (tid == 0) { s_prefix = 0; s_krem = K; s_whole = 0; }
   Key mask = 0;
   __syncthreads();
   // ---- radix select of the K-th smallest key, most significant digit first
@@ -95,9 +107,7 @@ __device__ void select_smallest_sorted(const Key* keys, int L, int K, int32_t* o
       }
       const int krem = s_krem;
       const int excl = incl - s;
-      const bool mine = excl < krem && krem <= incl;
-      const unsigned who = __ballot_sync(0xffffffffu, mine);
-      if (mine) {
+      if (excl < krem && krem <= incl) {
         int acc = excl, d = 0;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
@@ -106,29 +116,36 @@ __device__ void select_smallest_sorted(const Key* keys, int L, int K, int32_t* o
         }
         s_prefix = prefix | (Key(8 * tid + d) << shift);
         s_krem = krem - acc;
+        s_whole = c[d] == krem - acc;
       }
-      (void)who;
     }
     mask |= Key(0xff) << shift;
     __syncthreads();
+    if (s_whole) break;
   }
-  const Key T = s_prefix;      // the K-th smallest key
-  const int keep_eq = s_krem;  // how many keys equal to T are kept (lowest indices first)
-  // ---- ordered compaction: keep key < T, and the first keep_eq keys == T
-  int eq_base = 0, out_base = 0;
-  for (int base = 0; base < L; base += blockDim.x) {
-    const int i = base + tid;
-    const Key k = i < L ? keys[i] : Key(0);
-    const bool is_eq = i < L && k == T;
-    const int eq_rank = eq_base + block_excl_count(is_eq, warp_tot, &s_total);
-    const int eq_tot = s_total;
-    const bool keep = i < L && (k < T || (is_eq && eq_rank < keep_eq));
-    const int pos = out_base + block_excl_count(keep, warp_tot, &s_total);
-    const int keep_tot = s_total;
-    if (keep) out_idx[pos] = i;
-    eq_base += eq_tot;
-    out_base += keep_tot;
-    __syncthreads();
+  // keys are compared under `mask`: below the threshold T they are kept; equal
+  // to it, the first keep_eq of them (all of them when the select stopped early)
+  const Key T = s_prefix;
+  const int keep_eq = s_krem;
+  // ---- compaction over contiguous ranges of indices, one range per thread; an
+  // odd range length keeps a warp's reads of its 32 ranges on distinct banks
+  const int per = ((L + int(blockDim.x) - 1) / int(blockDim.x)) | 1;
+  const int i0 = min(L, tid * per), i1 = min(L, i0 + per);
+  int n_eq = 0;
+  for (int i = i0; i < i1; ++i) n_eq += (keys[i] & mask) == T;
+  int eq_rank = block_excl_sum(n_eq, warp_tot, &s_total);
+  int n_keep = 0;
+  for (int i = i0, r = eq_rank; i < i1; ++i) {
+    const Key km = keys[i] & mask;
+    if (km < T) ++n_keep;
+    else if (km == T) n_keep += r++ < keep_eq;
+  }
+  int pos = block_excl_sum(n_keep, warp_tot, &s_total);
+  for (int i = i0; i < i1; ++i) {
+    const Key km = keys[i] & mask;
+    bool keep = km < T;
+    if (km == T) keep = eq_rank++ < keep_eq;
+    if (keep) out_idx[pos++] = i;
   }
 }
 

@@ -8,7 +8,7 @@
 namespace sr {
 namespace {
 
-constexpr int BM = 64, BN = 64, BK = 16;
+constexpr int BN = 64, BK = 16;
 
 // Shared epilogue of every GEMM variant, applied to one output element.
 template <typename T, Epi E>
@@ -35,39 +35,62 @@ __device__ __forceinline__ void epilogue_store(const EpiArgs& ea, int m, int n, 
   }
 }
 
-template <typename T, Epi E>
+// four consecutive elements (16-byte aligned for fp32, 8-byte for bf16) as fp32
+__device__ __forceinline__ float4 load4(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
+__device__ __forceinline__ float4 load4(const bf16* p) {
+  const uint2 u = __ldg(reinterpret_cast<const uint2*>(p));
+  return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u),
+                     __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+}
+
+// BM x 64 output tile per CTA of 256 threads (BM = 64 or 32: 4 or 2 rows x 4
+// columns per thread); the 32-row tile doubles the CTAs of small GEMMs.  The
+// next k-slice of A and W is loaded into registers (4 consecutive k per load)
+// while the current one is multiplied from shared memory.
+template <typename T, Epi E, int BM>
 __global__ void __launch_bounds__(256)
 gemm_simt_kernel(const T* __restrict__ A, const T* __restrict__ W, int M, int N, int K,
                  EpiArgs ea) {
+  constexpr int RI = BM / 16;
   __shared__ float As[BK][BM + 4];
   __shared__ float Bs[BK][BN + 4];
   const int tid = threadIdx.x;
   const int tx = tid & 15, ty = tid >> 4;
   const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
-  float acc[4][4] = {};
+  float acc[RI][4] = {};
   const int lr = tid >> 2, lk = (tid & 3) * 4;   // loader: row lr, k lk..lk+3
+  const int am = m0 + lr, bn = n0 + lr;
+  const bool a_ok = lr < BM && am < M, b_ok = bn < N;
+  const T* ap = A + size_t(a_ok ? am : 0) * K + lk;
+  const T* bp = W + size_t(b_ok ? bn : 0) * K + lk;
+  const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+  float4 ra = a_ok ? load4(ap) : zero, rb = b_ok ? load4(bp) : zero;
   for (int k0 = 0; k0 < K; k0 += BK) {
-    const int am = m0 + lr, bn = n0 + lr;
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      As[lk + e][lr] = am < M ? Elem<T>::to_f(A[size_t(am) * K + k0 + lk + e]) : 0.f;
-      Bs[lk + e][lr] = bn < N ? Elem<T>::to_f(W[size_t(bn) * K + k0 + lk + e]) : 0.f;
+    if (lr < BM) {
+      As[lk][lr] = ra.x; As[lk + 1][lr] = ra.y; As[lk + 2][lr] = ra.z; As[lk + 3][lr] = ra.w;
     }
+    Bs[lk][lr] = rb.x; Bs[lk + 1][lr] = rb.y; Bs[lk + 2][lr] = rb.z; Bs[lk + 3][lr] = rb.w;
     __syncthreads();
+    if (k0 + BK < K) {
+      ra = a_ok ? load4(ap + k0 + BK) : zero;
+      rb = b_ok ? load4(bp + k0 + BK) : zero;
+    }
 #pragma unroll
     for (int k = 0; k < BK; ++k) {
-      float a[4], b[4];
+      float a[RI], b[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) { a[i] = As[k][ty + 16 * i]; b[i] = Bs[k][tx + 16 * i]; }
+      for (int i = 0; i < RI; ++i) a[i] = As[k][ty + 16 * i];
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
+      for (int i = 0; i < 4; ++i) b[i] = Bs[k][tx + 16 * i];
+#pragma unroll
+      for (int i = 0; i < RI; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
     }
     __syncthreads();
   }
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
+  for (int i = 0; i < RI; ++i) {
     const int m = m0 + ty + 16 * i;
     if (m >= M) continue;
 #pragma unroll
@@ -78,22 +101,30 @@ gemm_simt_kernel(const T* __restrict__ A, const T* __restrict__ W, int M, int N,
   }
 }
 
-// Attention core, one query row per thread, 128 rows per CTA, keys in tiles of
-// 32 staged in shared memory, online softmax (running max and sum) in fp32.
-constexpr int kAttRows = 128, kAttKeys = 32, kDh = 64;
+// Attention core: 16 query rows per CTA of 128 threads, each row's keys split
+// over 8 adjacent lanes (lane p of a row takes keys p, p + 8, ... of every
+// tile), keys and values staged in shared memory in tiles of 32, an online
+// softmax (running max and sum) per lane in fp32, and the 8 partial states of
+// a row merged by shuffles at the end:
+//   m = max_p m_p,  l = sum_p l_p 2^(m_p - m),  o = sum_p o_p 2^(m_p - m).
+constexpr int kAttRows = 16, kAttParts = 8, kAttThreads = kAttRows * kAttParts;
+constexpr int kAttKeys = 32, kDh = 64;
 
 template <typename T>
-__global__ void __launch_bounds__(kAttRows)
+__global__ void __launch_bounds__(kAttThreads)
 attention_simt_kernel(const T* __restrict__ qkv, T* __restrict__ out, int T_, int heads) {
-  __shared__ __align__(16) float Ks[kAttKeys][kDh];
-  __shared__ __align__(16) float Vs[kAttKeys][kDh];
+  // rows padded to 68 floats: the 8 keys a warp reads at once (one per lane
+  // part) start on 8 different 16-byte bank groups
+  __shared__ __align__(16) float Ks[kAttKeys][kDh + 4];
+  __shared__ __align__(16) float Vs[kAttKeys][kDh + 4];
   const int D = heads * kDh;
   const int ld = 3 * D;
   const int qtiles = (T_ + kAttRows - 1) / kAttRows;
   const int bh = blockIdx.x / qtiles;
   const int qt = blockIdx.x % qtiles;
   const int b = bh / heads, h = bh % heads;
-  const int row = qt * kAttRows + threadIdx.x;
+  const int part = threadIdx.x % kAttParts;
+  const int row = qt * kAttRows + threadIdx.x / kAttParts;
   const bool valid = row < T_;
   const T* base = qkv + size_t(b) * T_ * ld;
   // scores in the log2 domain: s * (1/sqrt(64)) * log2(e)
@@ -105,25 +136,37 @@ attention_simt_kernel(const T* __restrict__ qkv, T* __restrict__ out, int T_, in
     for (int d = 0; d < kDh; ++d) { q[d] = Elem<T>::to_f(qr[d]) * qscale; o[d] = 0.f; }
   }
   float mrun = -INFINITY, lrun = 0.f;
+  constexpr int kMine = kAttKeys / kAttParts;            // keys of a tile per lane
   for (int j0 = 0; j0 < T_; j0 += kAttKeys) {
     __syncthreads();
-    for (int e = threadIdx.x; e < kAttKeys * kDh; e += kAttRows) {
+    // the tile's keys and values, 4 consecutive elements per load; all of a
+    // thread's loads are issued before the first store
+    constexpr int kQuads = kAttKeys * kDh / 4 / kAttThreads;
+    float4 kq[kQuads], vq[kQuads];
+#pragma unroll
+    for (int u = 0; u < kQuads; ++u) {
+      const int e = 4 * (threadIdx.x + u * kAttThreads);
       const int j = e / kDh, d = e % kDh;
       const int key = j0 + j;
-      float kv = 0.f, vv = 0.f;
+      kq[u] = vq[u] = make_float4(0.f, 0.f, 0.f, 0.f);
       if (key < T_) {
-        const T* kr = base + size_t(key) * ld + D + h * kDh;
-        kv = Elem<T>::to_f(kr[d]);
-        vv = Elem<T>::to_f(kr[D + d]);
+        const T* kr = base + size_t(key) * ld + D + h * kDh + d;
+        kq[u] = load4(kr);
+        vq[u] = load4(kr + D);
       }
-      Ks[j][d] = kv;
-      Vs[j][d] = vv;
+    }
+#pragma unroll
+    for (int u = 0; u < kQuads; ++u) {
+      const int e = 4 * (threadIdx.x + u * kAttThreads);
+      *reinterpret_cast<float4*>(&Ks[e / kDh][e % kDh]) = kq[u];
+      *reinterpret_cast<float4*>(&Vs[e / kDh][e % kDh]) = vq[u];
     }
     __syncthreads();
-    float s[kAttKeys];
+    float s[kMine];
     float tmax = -INFINITY;
 #pragma unroll
-    for (int j = 0; j < kAttKeys; ++j) {
+    for (int i = 0; i < kMine; ++i) {
+      const int j = part + kAttParts * i;
       float acc = 0.f;
 #pragma unroll
       for (int d = 0; d < kDh; d += 4) {
@@ -131,17 +174,20 @@ attention_simt_kernel(const T* __restrict__ qkv, T* __restrict__ out, int T_, in
         acc = fmaf(q[d], k4.x, acc); acc = fmaf(q[d + 1], k4.y, acc);
         acc = fmaf(q[d + 2], k4.z, acc); acc = fmaf(q[d + 3], k4.w, acc);
       }
-      s[j] = (j0 + j < T_) ? acc : -INFINITY;
-      tmax = fmaxf(tmax, s[j]);
+      s[i] = (j0 + j < T_) ? acc : -INFINITY;
+      tmax = fmaxf(tmax, s[i]);
     }
+    // a lane whose keys so far all lie past the end keeps its empty state
+    if (tmax == -INFINITY) continue;
     const float mnew = fmaxf(mrun, tmax);
     const float corr = exp2f(mrun - mnew);
     lrun *= corr;
 #pragma unroll
     for (int d = 0; d < kDh; ++d) o[d] *= corr;
 #pragma unroll
-    for (int j = 0; j < kAttKeys; ++j) {
-      const float p = exp2f(s[j] - mnew);
+    for (int i = 0; i < kMine; ++i) {
+      const int j = part + kAttParts * i;
+      const float p = exp2f(s[i] - mnew);
       lrun += p;
 #pragma unroll
       for (int d = 0; d < kDh; d += 4) {
@@ -152,28 +198,58 @@ attention_simt_kernel(const T* __restrict__ qkv, T* __restrict__ out, int T_, in
     }
     mrun = mnew;
   }
+  // merge the row's 8 partial states (lanes 8r .. 8r+7 of the warp); every row
+  // has at least one key, so the merged max is finite
+  float m = mrun;
+#pragma unroll
+  for (int off = 1; off < kAttParts; off <<= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+  const float w = mrun == -INFINITY ? 0.f : exp2f(mrun - m);
+  float l = lrun * w;
+#pragma unroll
+  for (int off = 1; off < kAttParts; off <<= 1) l += __shfl_xor_sync(0xffffffffu, l, off);
+#pragma unroll
+  for (int d = 0; d < kDh; ++d) {
+    float v = o[d] * w;
+#pragma unroll
+    for (int off = 1; off < kAttParts; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    o[d] = v;
+  }
   if (valid) {
-    const float inv = 1.f / lrun;
+    // lane p of the row writes dimensions 8p .. 8p + 7
+    const float inv = 1.f / l;
     T* orow = out + (size_t(b) * T_ + row) * D + h * kDh;
 #pragma unroll
-    for (int d = 0; d < kDh; ++d) orow[d] = Elem<T>::from_f(o[d] * inv);
+    for (int d = 0; d < kDh; ++d)
+      if (d / (kDh / kAttParts) == part) orow[d] = Elem<T>::from_f(o[d] * inv);
   }
+}
+
+template <typename T, int BM>
+cudaError_t gemm_simt_bm(Epi epi, const void* A, const void* Bw, int M, int N, int K,
+                         const EpiArgs& ea, cudaStream_t s) {
+  dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM);
+  const T* a = static_cast<const T*>(A);
+  const T* w = static_cast<const T*>(Bw);
+  switch (epi) {
+    case Epi::Bias: gemm_simt_kernel<T, Epi::Bias, BM><<<grid, 256, 0, s>>>(a, w, M, N, K, ea); break;
+    case Epi::BiasGelu:
+      gemm_simt_kernel<T, Epi::BiasGelu, BM><<<grid, 256, 0, s>>>(a, w, M, N, K, ea); break;
+    case Epi::BiasResidual:
+      gemm_simt_kernel<T, Epi::BiasResidual, BM><<<grid, 256, 0, s>>>(a, w, M, N, K, ea); break;
+    case Epi::BiasResidualScatter:
+      gemm_simt_kernel<T, Epi::BiasResidualScatter, BM><<<grid, 256, 0, s>>>(a, w, M, N, K, ea);
+      break;
+  }
+  return cudaGetLastError();
 }
 
 template <typename T>
 cudaError_t gemm_simt_t(Epi epi, const void* A, const void* Bw, int M, int N, int K,
                         const EpiArgs& ea, cudaStream_t s) {
-  dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM);
-  const T* a = static_cast<const T*>(A);
-  const T* w = static_cast<const T*>(Bw);
-  switch (epi) {
-    case Epi::Bias: gemm_simt_kernel<T, Epi::Bias><<<grid, 256, 0, s>>>(a, w, M, N, K, ea); break;
-    case Epi::BiasGelu: gemm_simt_kernel<T, Epi::BiasGelu><<<grid, 256, 0, s>>>(a, w, M, N, K, ea); break;
-    case Epi::BiasResidual: gemm_simt_kernel<T, Epi::BiasResidual><<<grid, 256, 0, s>>>(a, w, M, N, K, ea); break;
-    case Epi::BiasResidualScatter:
-      gemm_simt_kernel<T, Epi::BiasResidualScatter><<<grid, 256, 0, s>>>(a, w, M, N, K, ea); break;
-  }
-  return cudaGetLastError();
+  // 64-row tiles when they already give two CTAs per SM, else 32-row tiles
+  const long ctas64 = long((N + BN - 1) / BN) * ((M + 63) / 64);
+  if (ctas64 >= 2 * 152) return gemm_simt_bm<T, 64>(epi, A, Bw, M, N, K, ea, s);
+  return gemm_simt_bm<T, 32>(epi, A, Bw, M, N, K, ea, s);
 }
 
 }  // namespace
@@ -189,11 +265,11 @@ cudaError_t launch_attention_simt(DType dt, const void* qkv, void* out, int B, i
                                   cudaStream_t s) {
   const int grid = B * heads * ((T + kAttRows - 1) / kAttRows);
   if (dt == DType::F32)
-    attention_simt_kernel<float><<<grid, kAttRows, 0, s>>>(static_cast<const float*>(qkv),
-                                                           static_cast<float*>(out), T, heads);
+    attention_simt_kernel<float><<<grid, kAttThreads, 0, s>>>(static_cast<const float*>(qkv),
+                                                              static_cast<float*>(out), T, heads);
   else
-    attention_simt_kernel<bf16><<<grid, kAttRows, 0, s>>>(static_cast<const bf16*>(qkv),
-                                                          static_cast<bf16*>(out), T, heads);
+    attention_simt_kernel<bf16><<<grid, kAttThreads, 0, s>>>(static_cast<const bf16*>(qkv),
+                                                             static_cast<bf16*>(out), T, heads);
   return cudaGetLastError();
 }
 
