@@ -54,7 +54,7 @@ constexpr uint32_t kColP = 384;    // P^t (bf16 pairs) at columns [384 + 64 t, 3
 constexpr float kRescaleLog2 = 8.0f;
 
 struct AttSmem {
-  uint64_t q_full;
+  uint64_t q_full, q_free;
   uint64_t k_full[kStages], k_empty[kStages], v_full[kStages], v_empty[kStages];
   uint64_t s_full[kQTiles], s_free[kQTiles], p_full[kQTiles], pv_done[kQTiles];
   uint64_t drain[1 + kQTiles];      // the S issuer, then each P V issuer
@@ -87,10 +87,18 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
   return d;
 }
 
+// kPersist: a CTA takes the work items (one (sample, head, 256-query block)
+// each) blockIdx.x, blockIdx.x + gridDim.x, ... in turn, with its barriers,
+// tensor memory and K/V rings kept across items; the next item's Q is loaded
+// once the previous item's S MMAs have read Q, and its first P V overwrites O
+// only after the previous item's epilogue has read O (the softmax threads read
+// O before they signal the next item's first P).  Without kPersist every CTA
+// has one item (the grid is the item count).
+template <bool kPersist>
 __global__ void __launch_bounds__(kThreads, 1)
 attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKV,
                     bf16* __restrict__ out, int Tq, int Tkv, int heads, int qcol0, int kcol0,
-                    int vcol0, unsigned int* fault) {
+                    int vcol0, int items, unsigned int* fault) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -101,15 +109,13 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qblocks = (Tq + kBQ - 1) / kBQ;
-  const int bh = blockIdx.x / qblocks;
-  const int qb = blockIdx.x % qblocks;
-  const int b = bh / heads, h = bh % heads;
   const int D = heads * kDh;
-  const int q0 = qb * kBQ;
   const int nkv = (Tkv + kKV - 1) / kKV;
+  const int item_step = kPersist ? int(gridDim.x) : items;
 
   if (threadIdx.x == 0) {
     mbar_init(&sm->q_full, 1);
+    mbar_init(&sm->q_free, 1);
     for (int s = 0; s < kStages; ++s) {
       // a K stage is released by the S issuer, a V stage by both P V issuers
       mbar_init(&sm->k_full[s], 1); mbar_init(&sm->k_empty[s], 1);
@@ -145,34 +151,44 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     asm volatile("setmaxnreg.dec.sync.aligned.u32 56;\n" ::: "memory");
     if (warp == 0) {
       // ------------------------------------------------------------- TMA loads
-      // the two Q tiles once, then K_j and V_j into their rings
+      // per item: the two Q tiles, then K_j and V_j into their rings
       if (lane == 0) {
-        mbar_arrive_expect_tx(&sm->q_full, kQTiles * kTileBytes);
-        for (int t = 0; t < kQTiles; ++t)
-          tma_load_3d(&tmQ, sQ + t * kTileBytes, &sm->q_full, qcol0 + h * kDh, q0 + t * kQTile, b);
-        const int kcol = kcol0 + h * kDh, vcol = vcol0 + h * kDh;
         // stages holding a load, and the parity of the phase each last used
         uint32_t kissued = 0, vissued = 0, kpar = 0, vpar = 0;
-        int st = 0;
+        int st = 0, q_loads = 0;
         uint32_t ph = 0;
-        for (int j = 0; j < nkv; ++j) {
-          // a K stage frees once both tiles' S MMAs of key tile j - kStages are done
-          if (!mbar_wait(&sm->k_empty[st], ph ^ 1, abort, fault)) break;
-          mbar_arrive_expect_tx(&sm->k_full[st], kTileBytes);
-          tma_load_3d(&tmKV, sK + st * kTileBytes, &sm->k_full[st], kcol, j * kKV, b);
-          kissued |= 1u << st;
-          kpar = (kpar & ~(1u << st)) | (ph << st);
-          // a V stage once both tiles' P V MMAs of that key tile are
-          if (!mbar_wait(&sm->v_empty[st], ph ^ 1, abort, fault)) break;
-          mbar_arrive_expect_tx(&sm->v_full[st], kTileBytes);
-          tma_load_3d(&tmKV, sV + st * kTileBytes, &sm->v_full[st], vcol, j * kKV, b);
-          vissued |= 1u << st;
-          vpar = (vpar & ~(1u << st)) | (ph << st);
-          if (++st == kStages) { st = 0; ph ^= 1; }
+        bool ok = true;
+        for (int item = blockIdx.x, it = 0; ok && item < items; item += item_step, ++it) {
+          const int bh = item / qblocks, qb = item % qblocks;
+          const int b = bh / heads, h = bh % heads;
+          // a persistent CTA reloads Q once the previous item's S MMAs have read it
+          if (kPersist && it > 0 && !(ok = mbar_wait(&sm->q_free, (it - 1) & 1, abort, fault))) break;
+          mbar_arrive_expect_tx(&sm->q_full, kQTiles * kTileBytes);
+          for (int t = 0; t < kQTiles; ++t)
+            tma_load_3d(&tmQ, sQ + t * kTileBytes, &sm->q_full, qcol0 + h * kDh,
+                        qb * kBQ + t * kQTile, b);
+          ++q_loads;
+          const int kcol = kcol0 + h * kDh, vcol = vcol0 + h * kDh;
+          for (int j = 0; j < nkv; ++j) {
+            // a K stage frees once both tiles' S MMAs of key tile j - kStages are done
+            if (!(ok = mbar_wait(&sm->k_empty[st], ph ^ 1, abort, fault))) break;
+            mbar_arrive_expect_tx(&sm->k_full[st], kTileBytes);
+            tma_load_3d(&tmKV, sK + st * kTileBytes, &sm->k_full[st], kcol, j * kKV, b);
+            kissued |= 1u << st;
+            kpar = (kpar & ~(1u << st)) | (ph << st);
+            // a V stage once both tiles' P V MMAs of that key tile are
+            if (!(ok = mbar_wait(&sm->v_empty[st], ph ^ 1, abort, fault))) break;
+            mbar_arrive_expect_tx(&sm->v_full[st], kTileBytes);
+            tma_load_3d(&tmKV, sV + st * kTileBytes, &sm->v_full[st], vcol, j * kKV, b);
+            vissued |= 1u << st;
+            vpar = (vpar & ~(1u << st)) | (ph << st);
+            if (++st == kStages) { st = 0; ph ^= 1; }
+          }
+          if constexpr (!kPersist) break;
         }
         // every issued load lands before the CTA may exit
         int no_abort = 0;
-        mbar_wait(&sm->q_full, 0, &no_abort, fault);
+        if (q_loads > 0) mbar_wait(&sm->q_full, uint32_t(q_loads - 1) & 1u, &no_abort, fault);
         for (int s = 0; s < kStages; ++s) {
           if (kissued & (1u << s)) mbar_wait(&sm->k_full[s], (kpar >> s) & 1u, &no_abort, fault);
           if (vissued & (1u << s)) mbar_wait(&sm->v_full[s], (vpar >> s) & 1u, &no_abort, fault);
@@ -180,30 +196,39 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
       }
     } else if (warp == 1) {
       // ------------------------------------------------------------- S MMAs
-      // S^t = Q^t K_j^T for both tiles, each once softmax t has read S^t of key
-      // tile j - 1
+      // S^t = Q^t K_j^T for both tiles, each once softmax t has read S^t of the
+      // previous key tile (of this item or, persistent, of the previous item)
       if (lane == 0) {
         constexpr uint32_t idesc_s = idesc_bf16(kQTile, kKV);                 // K-major A, B
-        bool ok = mbar_wait(&sm->q_full, 0, abort, fault);
-        int st = 0;
+        int st = 0, g = 0;                 // g: key tiles of earlier items
         uint32_t ph = 0;
-        for (int j = 0; j < nkv && ok; ++j) {
-          if (!(ok = mbar_wait(&sm->k_full[st], ph, abort, fault))) break;
-          const uint32_t ka = smem_u32(sK + st * kTileBytes);
-          for (int t = 0; t < kQTiles && ok; ++t) {
-            if (j > 0 && !(ok = mbar_wait(&sm->s_free[t], (j - 1) & 1, abort, fault))) break;
-            tc_fence_after();
-            const uint32_t qa = smem_u32(sQ + t * kTileBytes);
-            const uint32_t dS = tmem + kColS + uint32_t(t * kKV);
+        bool ok = true;
+        for (int item = blockIdx.x, it = 0; ok && item < items; item += item_step, ++it) {
+          const int gb = kPersist ? g : 0;
+          if (!(ok = mbar_wait(&sm->q_full, uint32_t(it) & 1u, abort, fault))) break;
+          for (int j = 0; j < nkv && ok; ++j) {
+            if (!(ok = mbar_wait(&sm->k_full[st], ph, abort, fault))) break;
+            const uint32_t ka = smem_u32(sK + st * kTileBytes);
+            for (int t = 0; t < kQTiles && ok; ++t) {
+              if (gb + j > 0 && !(ok = mbar_wait(&sm->s_free[t], (gb + j - 1) & 1, abort, fault))) break;
+              tc_fence_after();
+              const uint32_t qa = smem_u32(sQ + t * kTileBytes);
+              const uint32_t dS = tmem + kColS + uint32_t(t * kKV);
 #pragma unroll
-            for (int k = 0; k < kDh / 16; ++k)
-              mma_bf16(dS, sw128_desc(qa + 32 * k), sw128_desc(ka + 32 * k), idesc_s,
-                       k > 0 ? 1u : 0u);
-            mma_commit(&sm->s_full[t]);
+              for (int k = 0; k < kDh / 16; ++k)
+                mma_bf16(dS, sw128_desc(qa + 32 * k), sw128_desc(ka + 32 * k), idesc_s,
+                         k > 0 ? 1u : 0u);
+              mma_commit(&sm->s_full[t]);
+            }
+            if (!ok) break;
+            mma_commit(&sm->k_empty[st]);
+            if (++st == kStages) { st = 0; ph ^= 1; }
           }
           if (!ok) break;
-          mma_commit(&sm->k_empty[st]);
-          if (++st == kStages) { st = 0; ph ^= 1; }
+          // Q may be reloaded once this item's S MMAs are done
+          if constexpr (kPersist) mma_commit(&sm->q_free);
+          g += nkv;
+          if constexpr (!kPersist) break;
         }
         int no_abort = 0;
         mma_commit(&sm->drain[0]);
@@ -212,27 +237,34 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     } else {
       // ------------------------------------------------------------- P V MMAs
       // warp 2 for tile 0, warp 3 for tile 1: O^t += P^t_j V_j (128 x 64,
-      // accumulated in TMEM), P read from TMEM (64 columns of bf16 pairs)
+      // accumulated in TMEM), P read from TMEM (64 columns of bf16 pairs).  An
+      // item's first P V overwrites O; its P is signalled only after the
+      // softmax threads have read the previous item's O.
       if (lane == 0) {
         const int t = warp - 2;
         constexpr uint32_t idesc_o = idesc_bf16(kQTile, kDh, false, true);   // V is MN-major
         const uint32_t dO = tmem + kColO + uint32_t(t * kDh);
         const uint32_t aP = tmem + kColP + uint32_t(t * (kKV / 2));
         bool ok = true;
-        int st = 0;
+        int st = 0, g = 0;
         uint32_t ph = 0;
-        for (int j = 0; j < nkv && ok; ++j) {
-          if (!(ok = mbar_wait(&sm->v_full[st], ph, abort, fault))) break;
-          if (!(ok = mbar_wait(&sm->p_full[t], j & 1, abort, fault))) break;
-          tc_fence_after();
-          const uint32_t va = smem_u32(sV + st * kTileBytes);
+        for (int item = blockIdx.x; ok && item < items; item += item_step) {
+          const int gb = kPersist ? g : 0;
+          for (int j = 0; j < nkv && ok; ++j) {
+            if (!(ok = mbar_wait(&sm->v_full[st], ph, abort, fault))) break;
+            if (!(ok = mbar_wait(&sm->p_full[t], (gb + j) & 1, abort, fault))) break;
+            tc_fence_after();
+            const uint32_t va = smem_u32(sV + st * kTileBytes);
 #pragma unroll
-          for (int k = 0; k < kKV / 16; ++k)
-            mma_bf16_ts(dO, aP + uint32_t(k * 8), sw128_desc_mn(va + k * 2048), idesc_o,
-                        (j | k) != 0 ? 1u : 0u);
-          mma_commit(&sm->pv_done[t]);
-          mma_commit(&sm->v_empty[st]);
-          if (++st == kStages) { st = 0; ph ^= 1; }
+            for (int k = 0; k < kKV / 16; ++k)
+              mma_bf16_ts(dO, aP + uint32_t(k * 8), sw128_desc_mn(va + k * 2048), idesc_o,
+                          (j | k) != 0 ? 1u : 0u);
+            mma_commit(&sm->pv_done[t]);
+            mma_commit(&sm->v_empty[st]);
+            if (++st == kStages) { st = 0; ph ^= 1; }
+          }
+          g += nkv;
+          if constexpr (!kPersist) break;
         }
         int no_abort = 0;
         mma_commit(&sm->drain[1 + t]);
@@ -252,10 +284,16 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     const float c = 0.125f * 1.4426950408889634f;  // 1/sqrt(64) * log2(e)
     const float thresh = kRescaleLog2 / c;         // the same threshold in score units
     const uint64_t c2 = pk2(c, c);
-    float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
+    int g = 0;                                     // key tiles of earlier items
+    for (int item = blockIdx.x; ok && item < items; item += item_step) {
+    const int gb = kPersist ? g : 0;
+    const int bh = item / qblocks, qb = item % qblocks;
+    const int b = bh / heads, h = bh % heads;
+    const int q0 = qb * kBQ;
+    float m_run = -INFINITY, l_run = 0.f;
     for (int j = 0; j < nkv; ++j) {
-      ok = __all_sync(0xffffffffu, mbar_wait(&sm->s_full[t], j & 1, abort, fault));
+      ok = __all_sync(0xffffffffu, mbar_wait(&sm->s_full[t], (gb + j) & 1, abort, fault));
       if (!ok) break;
       tc_fence_after();
       // S with its row maximum: the load reduces each thread's 32 columns
@@ -319,8 +357,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
         l_run += (l0 + l1) + (l2 + l3);
       }
       // P and O of this tile are free once the previous P V has completed
-      if (j >= 1) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (j - 1) & 1, abort, fault));
+      if (gb + j >= 1) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (gb + j - 1) & 1, abort, fault));
         if (!ok) break;
         tc_fence_after();
       }
@@ -343,7 +381,7 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
       mbar_arrive(&sm->p_full[t]);
     }
     // epilogue: O / l for the rows that exist (the last P V implies all earlier ones)
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (nkv - 1) & 1, abort, fault));
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm->pv_done[t], (gb + nkv - 1) & 1, abort, fault));
     if (ok) {
       tc_fence_after();
       uint32_t o[2][32];
@@ -363,6 +401,9 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
                               pack_bf16x2(__uint_as_float(q[6]) * inv, __uint_as_float(q[7]) * inv));
         }
       }
+    }
+    g += nkv;
+    if constexpr (!kPersist) break;
     }
   }
   tc_fence_before();
@@ -403,23 +444,57 @@ cudaError_t make_map_btc(CUtensorMap* map, const void* ptr, int B, int T, uint64
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// Sets the kernel's attributes once and returns how many of its CTAs fit on the
+// GPU at once (one per SM: the CTA takes all 512 tensor-memory columns).
+template <bool kPersist>
+cudaError_t prepare(int* resident) {
+  static int cached = 0;
+  if (cached == 0) {
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, attention_tc_kernel<kPersist>);
+    if (e != cudaSuccess) return e;
+    if (fa.numRegs < 168) return cudaErrorInvalidConfiguration;   // the register split needs 168
+    e = cudaFuncSetAttribute(attention_tc_kernel<kPersist>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, int(kSmemBytes));
+    if (e != cudaSuccess) return e;
+    int dev = 0, sms = 0, per_sm = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attention_tc_kernel<kPersist>,
+                                                      kThreads, kSmemBytes);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    cached = sms * per_sm;
+  }
+  *resident = cached;
+  return cudaSuccess;
+}
+
+// Short key sequences (at most kPersistMaxKeyTiles key tiles) run on a
+// persistent grid of one CTA per SM: there a CTA's fixed cost (barrier setup,
+// tensor-memory allocation, the first loads, the epilogue and teardown, about
+// 3.3 us) is a large part of an item's work.  Longer ones run one CTA per item,
+// where the persistent loop's extra state costs more than it saves.
+constexpr int kPersistMaxKeyTiles = 16;
+
 cudaError_t launch(const CUtensorMap& tq, const CUtensorMap& tkv, void* out, int B, int Tq,
                    int Tkv, int heads, int qcol0, int kcol0, int vcol0, unsigned int* fault,
                    cudaStream_t s) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, attention_tc_kernel);
+  const int items = B * heads * ((Tq + kBQ - 1) / kBQ);
+  const int nkv = (Tkv + kKV - 1) / kKV;
+  int resident = 0;
+  if (nkv <= kPersistMaxKeyTiles) {
+    cudaError_t e = prepare<true>(&resident);
     if (e != cudaSuccess) return e;
-    if (fa.numRegs < 168) return cudaErrorInvalidConfiguration;   // the register split needs 168
-    e = cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             int(kSmemBytes));
-    if (e != cudaSuccess) return e;
-    attr_set = true;
+    if (items > resident)
+      return launch_k(attention_tc_kernel<true>, dim3(resident), dim3(kThreads), kSmemBytes, s, 1,
+                      tq, tkv, static_cast<bf16*>(out), Tq, Tkv, heads, qcol0, kcol0, vcol0, items,
+                      fault);
   }
-  const int grid = B * heads * ((Tq + kBQ - 1) / kBQ);
-  return launch_k(attention_tc_kernel, dim3(grid), dim3(kThreads), kSmemBytes, s, 1, tq, tkv,
-                  static_cast<bf16*>(out), Tq, Tkv, heads, qcol0, kcol0, vcol0, fault);
+  cudaError_t e = prepare<false>(&resident);
+  if (e != cudaSuccess) return e;
+  return launch_k(attention_tc_kernel<false>, dim3(items), dim3(kThreads), kSmemBytes, s, 1, tq, tkv,
+                  static_cast<bf16*>(out), Tq, Tkv, heads, qcol0, kcol0, vcol0, items, fault);
 }
 
 }  // namespace
