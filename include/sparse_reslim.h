@@ -147,7 +147,12 @@ sr_status sr_select(sr_handle* h, const void* x, float keep_ratio, uint64_t seed
  * baseline), with no selection, gather or scatter; n2 == 0 likewise routes
  * nothing.  Unselected rows of out are bit-identical to the input of the first
  * sparse block.  The delta of Eq. 9 is formed in fp32 from the last sparse
- * block's fp32 result and the stored h0, and x0 + delta is rounded once. */
+ * block's fp32 result and the stored h0, and x0 + delta is rounded once.
+ * CUDA graphs: the first call of a handle (and the first call of a shape in the
+ * process) sets kernel attributes and clears the handle's fault word; later
+ * calls only enqueue work on `stream`, so they can be captured into a CUDA
+ * graph and replayed (the keep ratio, seed and pointers are fixed in the
+ * graph). */
 sr_status sr_forward(sr_handle* h, const void* x, const sr_block_weights* w, float keep_ratio,
                      uint64_t seed, void* out, int32_t* idx_out, void* stream);
 

@@ -268,11 +268,23 @@ cudaError_t launch_token_laplacian(DType dt, const float* x, int B, int L, int g
                   score);
 }
 
+// Raises a kernel's dynamic shared-memory limit only when a launch needs more
+// than an earlier one set (so that calls after the first, which may be inside a
+// stream capture, make no attribute change).
+template <typename Kernel>
+static cudaError_t ensure_smem(Kernel kernel, size_t smem, int* current) {
+  if (int(smem) <= *current) return cudaSuccess;
+  const cudaError_t e =
+      cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e == cudaSuccess) *current = int(smem);
+  return e;
+}
+static int g_random_smem = 0, g_topk_smem = 0;
+
 cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared, int32_t* idx,
                                  cudaStream_t s) {
   const size_t smem = size_t(L) * sizeof(uint64_t);
-  cudaError_t e = cudaFuncSetAttribute(select_random_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  cudaError_t e = ensure_smem(select_random_kernel, smem, &g_random_smem);
   if (e != cudaSuccess) return e;
   return launch_k(select_random_kernel, dim3(B), dim3(kSelThreads), smem, s, 1, L, K, seed, shared,
                   idx);
@@ -281,8 +293,7 @@ cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared,
 cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t* idx,
                                cudaStream_t s, int parts) {
   const size_t smem = size_t(L) * sizeof(uint32_t);
-  cudaError_t e = cudaFuncSetAttribute(select_topk_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  cudaError_t e = ensure_smem(select_topk_kernel, smem, &g_topk_smem);
   if (e != cudaSuccess) return e;
   return launch_k(select_topk_kernel, dim3(B), dim3(kSelThreads), smem, s, 1, L, K, score, parts, idx);
 }

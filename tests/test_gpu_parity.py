@@ -316,3 +316,39 @@ def test_cross_attention_routed_over_full_sequence_sampled():
     ref = o.cross_attention(synth.stored_as_f64(q)[:, rows], synth.stored_as_f64(kv), heads)
     got = synth.stored_as_f64(out.cpu())[:, rows]
     check_parity("cross-attention 4050 over 16200, 52 sampled rows", got, ref, TOL["bf16"])
+
+
+# ------------------------------------------------------------ CUDA graphs
+@pytest.mark.parametrize("dtype,selector", [("bf16", "random"), ("bf16", "topk_l2"), ("f32", "random")])
+def test_forward_captured_in_a_cuda_graph_replays_bitwise(dtype, selector):
+    # after a first (warm-up) call, sr_forward only enqueues work: captured into a
+    # graph and replayed it gives bitwise the direct call's output, also after the
+    # input changes in place
+    from paper_2607_02829_gb300 import binding as b
+    wl = _tiny(dtype, B=2, L=256, heads=2, split=(1, 2, 1), r=0.25, selector=selector)
+    x, ws = synth.make_inputs(wl)
+    cfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, wl.n1, wl.n2, wl.n3, dtype=dtype,
+                        selector=selector)
+    enc = b.Encoder(cfg, max_keep_ratio=wl.keep_ratio)
+    xd = x.cuda()
+    wd = [{k: v.cuda() for k, v in blk.items()} for blk in ws]
+    warr = b.weights_array(wd)
+    ref, _ = enc.forward(xd, warr, wl.keep_ratio, 11)
+    out = torch.zeros_like(xd)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        b.sr_forward(enc.handle, xd.data_ptr(), warr, wl.keep_ratio, 11, out.data_ptr(), None,
+                     side.cuda_stream)
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(out, ref)
+    xd.mul_(0.5)
+    ref2, _ = enc.forward(xd, warr, wl.keep_ratio, 11)
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(out, ref2) and not torch.equal(ref2, ref)
+    assert b.sr_device_fault(enc.handle, False, torch.cuda.current_stream().cuda_stream) == 0
+    del g
+    enc.close()
