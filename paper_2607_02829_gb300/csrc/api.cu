@@ -89,7 +89,8 @@ size_t elem_size(int32_t dtype) { return dtype == SR_BF16 ? 2 : 4; }
 
 // Workspace layout for a config and a maximum routed count Kmax.
 struct Plan {
-  size_t fault, xs, ln, qkv, att, u, hs, idx, score, total;
+  size_t fault, xs, ln, qkv, att, u, hs, idx, score, splitk, total;
+  size_t splitk_floats;   // fp32 split-K scratch of the CUDA-core GEMMs (fp32 storage only)
   size_t block_rows;   // rows the per-block buffers (ln, qkv, att, u) hold
 };
 
@@ -114,6 +115,10 @@ Plan make_plan(const sr_config& c, int32_t Kmax) {
   // top-K scores: one per token, or the FC2 epilogue's partial sums per token
   const int parts = c.dtype == SR_BF16 ? std::max(1, sr::gemm_tc_sqnorm_parts(c.D)) : 1;
   p.score = off; off += align_up(rows * size_t(parts) * sizeof(float));
+  // the CUDA-core GEMMs split K in up to 8 slices when their output tiles alone
+  // leave SMs idle (the D-wide GEMMs of small row counts)
+  p.splitk_floats = c.dtype == SR_F32 ? 8 * brows * size_t(c.D) : 0;
+  p.splitk = off; off += align_up(p.splitk_floats * sizeof(float));
   p.total = off;
   return p;
 }
@@ -222,7 +227,8 @@ struct TraceScope {
 cudaError_t gemm(const sr_handle* h, Epi epi, const void* A, const void* W, int M, int N, int K,
                  const sr::EpiArgs& ea, cudaStream_t s) {
   if (h->dt == DType::BF16) return sr::launch_gemm_tc(epi, A, W, M, N, K, ea, s);
-  return sr::launch_gemm_simt(h->dt, epi, A, W, M, N, K, ea, s);
+  return sr::launch_gemm_simt(h->dt, epi, A, W, M, N, K, ea, s,
+                              static_cast<float*>(h->at(h->plan.splitk)), h->plan.splitk_floats);
 }
 
 cudaError_t attention(const sr_handle* h, const void* qkv, void* out, int B, int T,

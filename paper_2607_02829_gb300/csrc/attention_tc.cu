@@ -448,7 +448,10 @@ cudaError_t make_map_btc(CUtensorMap* map, const void* ptr, int B, int T, uint64
 // GPU at once (one per SM: the CTA takes all 512 tensor-memory columns).
 template <bool kPersist>
 cudaError_t prepare(int* resident) {
-  static int cached = 0;
+  static int cache[kMaxDevices] = {};
+  const int slot = device_slot();
+  if (slot < 0) return cudaErrorInvalidDevice;
+  int& cached = cache[slot];
   if (cached == 0) {
     cudaFuncAttributes fa;
     cudaError_t e = cudaFuncGetAttributes(&fa, attention_tc_kernel<kPersist>);

@@ -719,7 +719,6 @@ cudaError_t make_map_2d(CUtensorMap* map, const void* ptr, uint64_t rows, uint64
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-int g_num_sms = 0;
 
 // 2-D fp32 tensor map over a row-major [rows, cols] matrix, box [32, 32],
 // 128-byte swizzle (the residual stream tiles of the TMA epilogue).
@@ -758,21 +757,23 @@ cudaError_t launch_bn(const void* A, const void* W, int M, int N, int K, const E
     tr = tb;    // unused
   }
   auto kernel = gemm_tc_kernel<BN, E, kPair>;
-  static int max_units = 0;     // CTAs (or CTA pairs) resident at once
+  // CTAs (or CTA pairs) resident at once, per device
+  static int max_units_of[kMaxDevices] = {};
+  const int slot = device_slot();
+  if (slot < 0) return cudaErrorInvalidDevice;
+  int& max_units = max_units_of[slot];
   if (max_units == 0) {
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(C::kSmem));
     if (e != cudaSuccess) return e;
-    if (g_num_sms == 0) {
-      int dev = 0;
-      cudaGetDevice(&dev);
-      cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
-    }
+    int num_sms = 0;
+    e = cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, slot);
+    if (e != cudaSuccess) return e;
     if constexpr (kPair) {
       cudaLaunchConfig_t cfg = {};
       cudaLaunchAttribute at[1];
       at[0].id = cudaLaunchAttributeClusterDimension;
       at[0].val.clusterDim.x = 2; at[0].val.clusterDim.y = 1; at[0].val.clusterDim.z = 1;
-      cfg.gridDim = dim3(unsigned(g_num_sms & ~1));
+      cfg.gridDim = dim3(unsigned(num_sms & ~1));
       cfg.blockDim = dim3(kThreads);
       cfg.dynamicSmemBytes = C::kSmem;
       cfg.attrs = at;
@@ -783,7 +784,7 @@ cudaError_t launch_bn(const void* A, const void* W, int M, int N, int K, const E
       if (clusters < 1) return cudaErrorInvalidConfiguration;
       max_units = clusters;
     } else {
-      max_units = g_num_sms;
+      max_units = num_sms;
     }
   }
   const int tiles = ((M + C::kRowsTile - 1) / C::kRowsTile) * (N / BN);

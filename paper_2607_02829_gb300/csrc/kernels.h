@@ -51,6 +51,17 @@ inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
 }
 
+// ---- per-device caches of launch attributes -------------------------------
+// Kernel shared-memory limits and occupancy belong to a device's context, so
+// the launchers cache them per device ordinal (the current device).  Returns
+// -1 when the current device cannot be read or its ordinal is 64 or more.
+constexpr int kMaxDevices = 64;
+inline int device_slot() {
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= kMaxDevices) return -1;
+  return d;
+}
+
 // ---- token selection (Sec. 3.2; App. B.2) --------------------------------
 // Random: K smallest SplitMix64 keys per sample (ties by index), sorted indices.
 cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared,
@@ -123,8 +134,11 @@ struct EpiArgs {
 };
 // CUDA-core GEMM (fp32 storage) and tcgen05 GEMM (bf16 storage; K % 64 == 0,
 // N % 64 == 0).
+// splitk: optional fp32 scratch of splitk_floats for the partial sums of a
+// split-K launch (used when the output tiles alone would leave SMs idle).
 cudaError_t launch_gemm_simt(DType dt, Epi epi, const void* A, const void* Bw, int M, int N,
-                             int K, const EpiArgs& ea, cudaStream_t s);
+                             int K, const EpiArgs& ea, cudaStream_t s, float* splitk = nullptr,
+                             size_t splitk_floats = 0);
 cudaError_t launch_gemm_tc(Epi epi, const void* A, const void* Bw, int M, int N, int K,
                            const EpiArgs& ea, cudaStream_t s);
 // partial sums per row that launch_gemm_tc writes to EpiArgs::sqnorm for a

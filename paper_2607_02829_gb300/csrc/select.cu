@@ -279,12 +279,14 @@ static cudaError_t ensure_smem(Kernel kernel, size_t smem, int* current) {
   if (e == cudaSuccess) *current = int(smem);
   return e;
 }
-static int g_random_smem = 0, g_topk_smem = 0;
+static int g_random_smem[kMaxDevices] = {}, g_topk_smem[kMaxDevices] = {};
 
 cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared, int32_t* idx,
                                  cudaStream_t s) {
   const size_t smem = size_t(L) * sizeof(uint64_t);
-  cudaError_t e = ensure_smem(select_random_kernel, smem, &g_random_smem);
+  const int dev = device_slot();
+  if (dev < 0) return cudaErrorInvalidDevice;
+  cudaError_t e = ensure_smem(select_random_kernel, smem, &g_random_smem[dev]);
   if (e != cudaSuccess) return e;
   return launch_k(select_random_kernel, dim3(B), dim3(kSelThreads), smem, s, 1, L, K, seed, shared,
                   idx);
@@ -293,7 +295,9 @@ cudaError_t launch_select_random(int B, int L, int K, uint64_t seed, int shared,
 cudaError_t launch_select_topk(int B, int L, int K, const float* score, int32_t* idx,
                                cudaStream_t s, int parts) {
   const size_t smem = size_t(L) * sizeof(uint32_t);
-  cudaError_t e = ensure_smem(select_topk_kernel, smem, &g_topk_smem);
+  const int dev = device_slot();
+  if (dev < 0) return cudaErrorInvalidDevice;
+  cudaError_t e = ensure_smem(select_topk_kernel, smem, &g_topk_smem[dev]);
   if (e != cudaSuccess) return e;
   return launch_k(select_topk_kernel, dim3(B), dim3(kSelThreads), smem, s, 1, L, K, score, parts, idx);
 }

@@ -47,11 +47,16 @@ __device__ __forceinline__ float4 load4(const bf16* p) {
 // columns per thread); the 32-row tile doubles the CTAs of small GEMMs.  The
 // next k-slice of A and W is loaded into registers (4 consecutive k per load)
 // while the current one is multiplied from shared memory.
-template <typename T, Epi E, int BM>
+// kPart: split-K; CTA z of the grid's third dimension multiplies the K / gridDim.z
+// columns from z * K / gridDim.z on and stores its raw sums in part[z][M][N]
+// (the epilogue runs in splitk_epilogue_kernel).
+template <typename T, Epi E, int BM, bool kPart = false>
 __global__ void __launch_bounds__(256)
 gemm_simt_kernel(const T* __restrict__ A, const T* __restrict__ W, int M, int N, int K,
-                 EpiArgs ea) {
+                 EpiArgs ea, float* __restrict__ part = nullptr) {
   constexpr int RI = BM / 16;
+  const int Kc = kPart ? K / int(gridDim.z) : K;          // columns of K this CTA multiplies
+  const int kz = kPart ? int(blockIdx.z) * Kc : 0;
   __shared__ float As[BK][BM + 4];
   __shared__ float Bs[BK][BN + 4];
   const int tid = threadIdx.x;
@@ -61,17 +66,17 @@ gemm_simt_kernel(const T* __restrict__ A, const T* __restrict__ W, int M, int N,
   const int lr = tid >> 2, lk = (tid & 3) * 4;   // loader: row lr, k lk..lk+3
   const int am = m0 + lr, bn = n0 + lr;
   const bool a_ok = lr < BM && am < M, b_ok = bn < N;
-  const T* ap = A + size_t(a_ok ? am : 0) * K + lk;
-  const T* bp = W + size_t(b_ok ? bn : 0) * K + lk;
+  const T* ap = A + size_t(a_ok ? am : 0) * K + kz + lk;
+  const T* bp = W + size_t(b_ok ? bn : 0) * K + kz + lk;
   const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
   float4 ra = a_ok ? load4(ap) : zero, rb = b_ok ? load4(bp) : zero;
-  for (int k0 = 0; k0 < K; k0 += BK) {
+  for (int k0 = 0; k0 < Kc; k0 += BK) {
     if (lr < BM) {
       As[lk][lr] = ra.x; As[lk + 1][lr] = ra.y; As[lk + 2][lr] = ra.z; As[lk + 3][lr] = ra.w;
     }
     Bs[lk][lr] = rb.x; Bs[lk + 1][lr] = rb.y; Bs[lk + 2][lr] = rb.z; Bs[lk + 3][lr] = rb.w;
     __syncthreads();
-    if (k0 + BK < K) {
+    if (k0 + BK < Kc) {
       ra = a_ok ? load4(ap + k0 + BK) : zero;
       rb = b_ok ? load4(bp + k0 + BK) : zero;
     }
@@ -96,8 +101,26 @@ gemm_simt_kernel(const T* __restrict__ A, const T* __restrict__ W, int M, int N,
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const int n = n0 + tx + 16 * j;
-      if (n < N) epilogue_store<T, E>(ea, m, n, N, acc[i][j]);
+      if (n >= N) continue;
+      if constexpr (kPart)
+        part[(size_t(blockIdx.z) * M + m) * N + n] = acc[i][j];
+      else
+        epilogue_store<T, E>(ea, m, n, N, acc[i][j]);
     }
+  }
+}
+
+// The split-K sums part[0] + part[1] + ... (in slice order) and the fused
+// epilogue, one output element per thread.
+template <typename T, Epi E>
+__global__ void __launch_bounds__(256)
+splitk_epilogue_kernel(const float* __restrict__ part, int S, int M, int N, EpiArgs ea) {
+  const size_t MN = size_t(M) * N;
+  for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < MN;
+       i += size_t(gridDim.x) * blockDim.x) {
+    float acc = part[i];
+    for (int z = 1; z < S; ++z) acc += part[size_t(z) * MN + i];
+    epilogue_store<T, E>(ea, int(i / N), int(i % N), N, acc);
   }
 }
 
@@ -243,22 +266,51 @@ cudaError_t gemm_simt_bm(Epi epi, const void* A, const void* Bw, int M, int N, i
   return cudaGetLastError();
 }
 
+template <typename T, Epi E>
+cudaError_t gemm_simt_splitk(const T* a, const T* w, int M, int N, int K, int S,
+                             const EpiArgs& ea, float* part, cudaStream_t s) {
+  dim3 grid((N + BN - 1) / BN, (M + 31) / 32, S);
+  gemm_simt_kernel<T, E, 32, true><<<grid, 256, 0, s>>>(a, w, M, N, K, ea, part);
+  const size_t MN = size_t(M) * N;
+  const int blocks = int((MN + 255) / 256 < 152 * 8 ? (MN + 255) / 256 : 152 * 8);
+  splitk_epilogue_kernel<T, E><<<blocks, 256, 0, s>>>(part, S, M, N, ea);
+  return cudaGetLastError();
+}
+
 template <typename T>
 cudaError_t gemm_simt_t(Epi epi, const void* A, const void* Bw, int M, int N, int K,
-                        const EpiArgs& ea, cudaStream_t s) {
-  // 64-row tiles when they already give two CTAs per SM, else 32-row tiles
+                        const EpiArgs& ea, cudaStream_t s, float* part, size_t part_floats) {
+  // 64-row tiles when they already give two CTAs per SM, else 32-row tiles;
+  // when even those leave SMs idle, K is split into S slices (a power of two,
+  // at most 8, each at least 128 columns) that run side by side
   const long ctas64 = long((N + BN - 1) / BN) * ((M + 63) / 64);
   if (ctas64 >= 2 * 152) return gemm_simt_bm<T, 64>(epi, A, Bw, M, N, K, ea, s);
+  const long ctas32 = long((N + BN - 1) / BN) * ((M + 31) / 32);
+  int S = 1;
+  while (ctas32 * S < 2 * 152 && S < 8 && K % (2 * S * BK) == 0 && K / (2 * S) >= 128) S *= 2;
+  if (S > 1 && part && size_t(S) * M * N <= part_floats) {
+    const T* a = static_cast<const T*>(A);
+    const T* w = static_cast<const T*>(Bw);
+    switch (epi) {
+      case Epi::Bias: return gemm_simt_splitk<T, Epi::Bias>(a, w, M, N, K, S, ea, part, s);
+      case Epi::BiasGelu: return gemm_simt_splitk<T, Epi::BiasGelu>(a, w, M, N, K, S, ea, part, s);
+      case Epi::BiasResidual:
+        return gemm_simt_splitk<T, Epi::BiasResidual>(a, w, M, N, K, S, ea, part, s);
+      case Epi::BiasResidualScatter:
+        return gemm_simt_splitk<T, Epi::BiasResidualScatter>(a, w, M, N, K, S, ea, part, s);
+    }
+  }
   return gemm_simt_bm<T, 32>(epi, A, Bw, M, N, K, ea, s);
 }
 
 }  // namespace
 
 cudaError_t launch_gemm_simt(DType dt, Epi epi, const void* A, const void* Bw, int M, int N,
-                             int K, const EpiArgs& ea, cudaStream_t s) {
+                             int K, const EpiArgs& ea, cudaStream_t s, float* splitk,
+                             size_t splitk_floats) {
   if (ea.sqnorm) return cudaErrorInvalidValue;     // row norms are fused on the tcgen05 path only
-  if (dt == DType::F32) return gemm_simt_t<float>(epi, A, Bw, M, N, K, ea, s);
-  return gemm_simt_t<bf16>(epi, A, Bw, M, N, K, ea, s);
+  if (dt == DType::F32) return gemm_simt_t<float>(epi, A, Bw, M, N, K, ea, s, splitk, splitk_floats);
+  return gemm_simt_t<bf16>(epi, A, Bw, M, N, K, ea, s, splitk, splitk_floats);
 }
 
 cudaError_t launch_attention_simt(DType dt, const void* qkv, void* out, int B, int T, int heads,
