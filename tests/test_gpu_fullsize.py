@@ -5,6 +5,8 @@
   tests/golden/ (written by tests/golden/make_c4_golden.py, which calls only
   the oracle) as a quick check, then the whole oracle forward element by
   element; the bit-exact index set and unselected-row passthrough.
+* 0.25 deg Laplacian selection, and the implicit ensemble at the 5.625 deg bf16
+  size (members bitwise sr_forward, the mean within rounding of theirs).
 * keep-ratio x selector sweep on the 1.40625 deg model (random, top-K L2 norm,
   and the Laplacian selector): index sets for every point, r = 1 bitwise equal
   to the dense stack, and the whole output against the oracle at every point of
@@ -160,3 +162,51 @@ def test_sweep_forward_matches_oracle(sweep_inputs, sweep_oracle_early, selector
                            seed=wl.select_seed, idx=None if selector == "random" else idx,
                            threads=THREADS)
     check_parity(f"{wl.name} (full output)", synth.stored_as_f64(out), ref, TOL)
+
+
+def test_c4_laplacian_selection_matches_oracle():
+    # the Laplacian selector on the 0.25 deg patch grid (90 x 180 tokens): the
+    # GPU's index set against the oracle's on the GPU's own pre-routing state,
+    # equal up to the fp32 tie band, and the unselected rows passed through
+    wl = synth.WORKLOADS["c4_0p25deg_bf16"].with_(selector="laplacian")
+    x, ws = synth.make_inputs(wl)
+    K = o.keep_count(wl.L, wl.keep_ratio)
+    _, idx = gpu_forward(wl, x, ws, n_split=(wl.n1, wl.n2, 0))
+    ok, pre = _passthrough_ok(wl, x, ws, idx)
+    assert ok
+    x0 = synth.stored_as_f64(pre)
+    s = o.token_laplacian_scores(x0, wl.grid_wp)
+    exp = o.select_topk_laplacian(x0, K, wl.grid_wp)
+    kth = np.sort(s[0])[::-1][K - 1]
+    diff = set(idx[0].tolist()) ^ set(exp[0].tolist())
+    assert len(diff) <= 8 and all(abs(s[0, i] - kth) <= 1e-5 * kth for i in diff), sorted(diff)
+
+
+def test_c2_ensemble_members_bitwise_and_mean():
+    # the implicit ensemble at the 5.625 deg bf16 size (B = 32): the members run
+    # as one batch of 64 samples; each is bitwise sr_forward with its seed, and
+    # the mean is the members' fp32 mean rounded once (within one bf16 ulp of
+    # the fp64 mean of the stored members)
+    from paper_2607_02829_gb300 import binding as b
+    wl = synth.WORKLOADS["c2_5p625deg_bf16"]
+    x, ws = synth.make_inputs(wl)
+    cfg = b.make_config(wl.B, wl.L, wl.D, wl.heads, wl.n1, wl.n2, wl.n3, dtype="bf16")
+    enc = b.Encoder(cfg, max_keep_ratio=wl.keep_ratio)
+    xd = x.cuda()
+    wd = [{k: v.cuda() for k, v in blk.items()} for blk in ws]
+    warr = b.weights_array(wd)
+    seeds = [5, 2**40 + 1]
+    mean, members, idx = enc.forward_ensemble(xd, warr, wl.keep_ratio, seeds, want_members=True,
+                                              want_idx=True)
+    for m, sd in enumerate(seeds):
+        y, i1 = enc.forward(xd, warr, wl.keep_ratio, sd, want_idx=True)
+        assert torch.equal(members[m], y) and torch.equal(idx[m], i1)
+    torch.cuda.synchronize()
+    mem = synth.stored_as_f64(members.cpu())
+    mf = mem.mean(axis=0)
+    got = synth.stored_as_f64(mean.cpu())
+    # each stored member is its fp32 value rounded to bf16 (within 2^-9 of it,
+    # relatively), and the mean is rounded once more
+    bound = 2.0 ** -8 * (np.abs(mem).mean(axis=0) + np.abs(mf))
+    assert np.all(np.abs(got - mf) <= bound)
+    enc.close()
