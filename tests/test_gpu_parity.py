@@ -139,6 +139,7 @@ def test_in_place_equals_out_of_place():
     ("bf16", 1, 1, 1, (1, 1, 1), 1.0),        # a single token
     ("bf16", 2, 129, 2, (0, 2, 0), 0.125),    # K = 16, routing only
     ("f32", 1, 97, 1, (2, 1, 0), 0.5),
+    ("bf16", 2, 129, 2, (1, 1, 1), 0.0078125),  # K = 1: one routed token per sample
 ])
 def test_forward_parity_small(dtype, B, L, heads, split, r):
     wl = _tiny(dtype, B=B, L=L, heads=heads, split=split, r=r)
@@ -149,6 +150,19 @@ def test_forward_parity_small(dtype, B, L, heads, split, r):
         assert np.array_equal(idx, ridx)
     check_parity(f"small {dtype} B={B} L={L} H={heads} split={split} r={r}",
                  synth.stored_as_f64(out), ref, TOL[dtype])
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_forward_parity_shared_index_set(dtype):
+    # one index set for the whole batch (the App. A.4 listing's reading)
+    wl = _tiny(dtype, B=3, L=200, heads=2, split=(1, 2, 1), r=0.25)
+    x, ws = synth.make_inputs(wl)
+    out, idx = gpu_forward(wl, x, ws, shared=True)
+    assert all(np.array_equal(idx[0], idx[i]) for i in range(wl.B))
+    ref, ridx = o.forward(synth.stored_as_f64(x), o.as_f64_weights(ws), 1, 2, 1, wl.heads,
+                          wl.keep_ratio, seed=wl.select_seed, shared_indices=True, threads=8)
+    assert np.array_equal(idx, ridx)
+    check_parity(f"small {dtype} shared index set", synth.stored_as_f64(out), ref, TOL[dtype])
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])

@@ -312,15 +312,20 @@ CASES = [
     ("top-K keeps the smallest norms", {"select_topk_l2": m_topk_smallest},
      ["test_topk_bruteforce_with_ties"]),
     ("Laplacian: latitude wraps around", {"token_laplacian_scores": m_lap_lat_periodic},
-     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce"]),
+     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce",
+      "test_laplacian_scores_against_scipy_ndimage"]),
     ("Laplacian: zero outside the poles", {"token_laplacian_scores": m_lap_lat_zero},
-     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce"]),
+     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce",
+      "test_laplacian_scores_against_scipy_ndimage"]),
     ("Laplacian: longitude reflected, not periodic", {"token_laplacian_scores": m_lap_lon_reflected},
-     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce"]),
+     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce",
+      "test_laplacian_scores_against_scipy_ndimage"]),
     ("Laplacian: centre weight 2", {"token_laplacian_scores": m_lap_centre_two},
-     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce"]),
+     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce",
+      "test_laplacian_scores_against_scipy_ndimage"]),
     ("Laplacian: grid rows and columns swapped", {"token_laplacian_scores": m_lap_grid_transposed},
-     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce"]),
+     ["test_laplacian_scores_closed_forms", "test_laplacian_scores_bruteforce",
+      "test_laplacian_scores_against_scipy_ndimage"]),
     ("Laplacian top-K ties to the higher index", {"select_topk_laplacian": m_lap_topk_ties_high},
      ["test_laplacian_topk_bruteforce_with_ties"]),
     ("LayerNorm with the unbiased variance", {"layer_norm": m_ln_unbiased},

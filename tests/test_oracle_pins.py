@@ -177,6 +177,21 @@ def test_laplacian_scores_bruteforce():
                            rtol=1e-13, atol=1e-13)
 
 
+def test_laplacian_scores_against_scipy_ndimage():
+    # scipy's discrete Laplacian over the two grid axes, latitude edges repeated
+    # ("nearest": x(-1) = x(0)) and longitude periodic ("wrap"), squared and
+    # summed over the features
+    ndimage = pytest.importorskip("scipy.ndimage")
+    rng = np.random.default_rng(23)
+    for (B, H, W, D) in [(2, 6, 9, 5), (1, 90, 180, 4), (1, 3, 2, 3)]:
+        x = rng.standard_normal((B, H * W, D))
+        for b in range(B):
+            lap = ndimage.laplace(x[b].reshape(H, W, D), mode=["nearest", "wrap"], axes=(0, 1))
+            expect = (lap ** 2).sum(axis=-1).reshape(-1)
+            assert np.allclose(o.token_laplacian_scores(x[b:b + 1], W)[0], expect,
+                               rtol=1e-12, atol=1e-12)
+
+
 def test_laplacian_topk_bruteforce_with_ties():
     rng = np.random.default_rng(5)
     H, W = 4, 5
