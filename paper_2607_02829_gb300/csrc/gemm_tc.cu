@@ -68,6 +68,16 @@ struct GemmCfg {
                 : size_t(kEpiThreads / 32) * kStageFloats * 4;
   static constexpr size_t kSmem =
       size_t(kStages) * kStageBytes + kStagingBytes + 1024 /*align*/ + 512 /*barriers*/;
+  // delta scatter on a unit's last tile: each epilogue warp stages 32-column
+  // quarters of its routed rows h and of the stream rows x0 (4 KB each) in the
+  // then idle operand ring, up to three quarters in flight
+  static constexpr int kScatterQuarters = BN / 64;                  // per warp
+  static constexpr int kScatterSlots = kScatterQuarters < 3 ? kScatterQuarters : 3;
+  static constexpr int kScatterSlotBytes = 2 * 32 * 32 * 4;
+  static_assert(E != Epi::BiasResidualScatter ||
+                    size_t(kEpiThreads / 32) * kScatterSlots * kScatterSlotBytes <=
+                        size_t(kStages) * kStageBytes,
+                "scatter staging exceeds the operand ring");
 };
 
 struct Smem {
@@ -107,6 +117,22 @@ __device__ __forceinline__ void gelu2_as7126(float& z0, float& z1) {
 
 __device__ __forceinline__ void prefetch_l2(const void* p) {
   asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
+// 16-byte copy from global to shared memory through L2 only (cp.async.cg);
+// each thread's copies complete in commit groups it waits for
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem)), "l"(gmem)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+// waits until at most n of this thread's commit groups are still in flight (n < 3)
+__device__ __forceinline__ void cp_async_wait_upto(int n) {
+  if (n <= 0) asm volatile("cp.async.wait_group 0;" ::: "memory");
+  else if (n == 1) asm volatile("cp.async.wait_group 1;" ::: "memory");
+  else asm volatile("cp.async.wait_group 2;" ::: "memory");
 }
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
@@ -574,13 +600,17 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         }
       } else if constexpr (E == Epi::BiasResidualScatter) {
         // last sparse block: hn = h + f(h); x'[xrow] = x0 + (hn - x0), h0 == x0.
-        // The warp walks its 32 rows x BN/2 columns in steps of 16 rows x 32
-        // columns.  A step's global loads (the routed rows h and the stream rows
-        // x0 they scatter into, 128 contiguous bytes per row) are issued one step
-        // ahead, the first step's before the accumulator is ready, so a step waits
-        // for at most one round trip and its stores overlap the next step's
-        // loads.  Element offsets fit 32 bits: sr_create rejects B * L * width
-        // >= 2^31.
+        // Every row the warp reads (the routed rows h and the stream rows x0
+        // they scatter into, 128 contiguous bytes per row and 32 columns) is
+        // prefetched into L2 while the mainloop runs.  On the unit's last tile
+        // the rows are then copied into the idle operand ring, three 32-column
+        // quarters at once; on earlier tiles (the ring is still in use) the warp
+        // walks its 32 rows x BN/2 columns in steps of 16 rows x 32 columns with
+        // each step's loads issued one step ahead.  Either way a thread owns one
+        // column of a row at a time (through the per-warp transpose buffer), so
+        // every store of a row covers 128 contiguous bytes, and the arithmetic is
+        // the same.  Element offsets fit 32 bits: sr_create rejects B * L *
+        // width >= 2^31.
         constexpr int kSteps = 2 * (BN / 64);
         const int m_lane = row0 + lane;
         const uint32_t xrow_lane =
@@ -611,37 +641,95 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             prefetch_l2(xp + 128 * l);
           }
         }
-        float rv[2][16], x0[2][16];
-        load_step(0, rv[0], x0[0]);
-        if (!__all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault))) break;
-        tc_fence_after();
-        const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
-        float* stg = staging + (warp - 2) * C::kStageFloats;
+        if (t + units >= tiles) {
+          // the unit's last tile: once the accumulator is ready no MMA reads the
+          // operand ring and no load refills it, so each warp stages there the
+          // rows it updates, a 32-column quarter at a time (its routed rows h
+          // and the stream rows x0), with up to three quarters in flight
+          if (!__all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault))) break;
+          tc_fence_after();
+          fence_proxy_async_smem();      // the ring was last written and read by the async proxy
+          unsigned char* wbuf = sA + size_t(warp - 2) * C::kScatterSlots * C::kScatterSlotBytes;
+          auto fetch = [&](int k) {
+            unsigned char* hb = wbuf + (k % C::kScatterSlots) * C::kScatterSlotBytes;
+            const int col = nt * BN + c_begin + 32 * k + 4 * (lane & 7);
 #pragma unroll
-        for (int st = 0; st < kSteps; ++st) {
-          const int c = c_begin + 32 * (st >> 1);
-          if ((st & 1) == 0) {
-            // this thread's row of the chunk's accumulators into the transpose buffer
+            for (int rr = 0; rr < 8; ++rr) {
+              const int i = (lane >> 3) + 4 * rr;      // 4 rows x 128 bytes per instruction
+              const uint32_t xr = __shfl_sync(0xffffffffu, xrow_lane, i);
+              if (row0 + i < M) {
+                cp_async16(hb + i * 128 + (lane & 7) * 16, hres + size_t(row0 + i) * N + col);
+                cp_async16(hb + 4096 + i * 128 + (lane & 7) * 16, xs + xr + uint32_t(col));
+              }
+            }
+            cp_async_commit();
+          };
+#pragma unroll
+          for (int k = 0; k < C::kScatterSlots; ++k) fetch(k);
+          const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
+          float* stg = staging + (warp - 2) * C::kStageFloats;
+#pragma unroll 1
+          for (int k = 0; k < C::kScatterQuarters; ++k) {
+            const int c = c_begin + 32 * k;
             uint32_t r[32];
             tmem_ld32(tbase + uint32_t(c), r);
             tmem_wait_ld();
 #pragma unroll
             for (int j = 0; j < 32; ++j) stg[lane * 33 + j] = __uint_as_float(r[j]);
+            // quarter k has landed once at most the later ones are in flight
+            const int issued = min(C::kScatterQuarters, k + C::kScatterSlots);
+            cp_async_wait_upto(issued - (k + 1));
             __syncwarp();
-          }
-          if (st + 1 < kSteps) load_step(st + 1, rv[(st + 1) & 1], x0[(st + 1) & 1]);
-          const int col = nt * BN + c + lane;
-          const float bias = __bfloat162float(static_cast<const bf16*>(ea.bias)[col]);
-          const int i0 = 16 * (st & 1);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const uint32_t xr = __shfl_sync(0xffffffffu, xrow_lane, i0 + i);
-            if (row0 + i0 + i < M) {
-              const float hn = rv[st & 1][i] + (stg[(i0 + i) * 33 + lane] + bias);
-              xs[xr + uint32_t(col)] = x0[st & 1][i] + (hn - x0[st & 1][i]);
+            const float* hq =
+                reinterpret_cast<const float*>(wbuf + (k % C::kScatterSlots) * C::kScatterSlotBytes);
+            const float* xq = hq + 32 * 32;
+            const int col = nt * BN + c + lane;
+            const float bias = __bfloat162float(static_cast<const bf16*>(ea.bias)[col]);
+#pragma unroll 4
+            for (int i = 0; i < 32; ++i) {
+              const uint32_t xr = __shfl_sync(0xffffffffu, xrow_lane, i);
+              if (row0 + i < M) {
+                const float hn = hq[i * 32 + lane] + (stg[i * 33 + lane] + bias);
+                const float x0v = xq[i * 32 + lane];
+                xs[xr + uint32_t(col)] = x0v + (hn - x0v);
+              }
             }
+            __syncwarp();                // the slot and the transpose buffer are rewritten next
+            if (k + C::kScatterSlots < C::kScatterQuarters) fetch(k + C::kScatterSlots);
           }
-          if (st & 1) __syncwarp();      // the next chunk rewrites the transpose buffer
+        } else {
+          float rv[2][16], x0[2][16];
+          load_step(0, rv[0], x0[0]);
+          if (!__all_sync(0xffffffffu, mbar_wait<kPair>(&sm->tfull[acc], aphase, abort, ea.fault))) break;
+          tc_fence_after();
+          const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
+          float* stg = staging + (warp - 2) * C::kStageFloats;
+  #pragma unroll
+          for (int st = 0; st < kSteps; ++st) {
+            const int c = c_begin + 32 * (st >> 1);
+            if ((st & 1) == 0) {
+              // this thread's row of the chunk's accumulators into the transpose buffer
+              uint32_t r[32];
+              tmem_ld32(tbase + uint32_t(c), r);
+              tmem_wait_ld();
+  #pragma unroll
+              for (int j = 0; j < 32; ++j) stg[lane * 33 + j] = __uint_as_float(r[j]);
+              __syncwarp();
+            }
+            if (st + 1 < kSteps) load_step(st + 1, rv[(st + 1) & 1], x0[(st + 1) & 1]);
+            const int col = nt * BN + c + lane;
+            const float bias = __bfloat162float(static_cast<const bf16*>(ea.bias)[col]);
+            const int i0 = 16 * (st & 1);
+  #pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              const uint32_t xr = __shfl_sync(0xffffffffu, xrow_lane, i0 + i);
+              if (row0 + i0 + i < M) {
+                const float hn = rv[st & 1][i] + (stg[(i0 + i) * 33 + lane] + bias);
+                xs[xr + uint32_t(col)] = x0[st & 1][i] + (hn - x0[st & 1][i]);
+              }
+            }
+            if (st & 1) __syncwarp();      // the next chunk rewrites the transpose buffer
+          }
         }
       } else {
         // the first chunk's residual loads overlap the wait for the accumulator
