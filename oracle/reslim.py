@@ -8,7 +8,7 @@ library primitive.
 
 What it computes (arxiv 2607.02829):
 
-* K = floor(L * r)                                   -- Sec. 3.2, Alg. 1 line "K <- ..."
+* K = floor(L * r)                                   -- Sec. 3.2, Alg. 1
 * the three-stage block partition (n1 dense, n2 sparse, n3 dense) -- Sec. 3.2 Eq. 7
 * token selection, uniform without replacement, sorted ascending  -- Sec. 3.2
   (the paper draws it with torch.randperm, which cannot be reproduced
