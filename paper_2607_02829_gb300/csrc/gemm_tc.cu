@@ -704,7 +704,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           tc_fence_after();
           const uint32_t tbase = tmem + (uint32_t(q * 32) << 16) + uint32_t(acc * BN);
           float* stg = staging + (warp - 2) * C::kStageFloats;
-  #pragma unroll
+#pragma unroll
           for (int st = 0; st < kSteps; ++st) {
             const int c = c_begin + 32 * (st >> 1);
             if ((st & 1) == 0) {
@@ -712,7 +712,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               uint32_t r[32];
               tmem_ld32(tbase + uint32_t(c), r);
               tmem_wait_ld();
-  #pragma unroll
+#pragma unroll
               for (int j = 0; j < 32; ++j) stg[lane * 33 + j] = __uint_as_float(r[j]);
               __syncwarp();
             }
@@ -720,7 +720,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             const int col = nt * BN + c + lane;
             const float bias = __bfloat162float(static_cast<const bf16*>(ea.bias)[col]);
             const int i0 = 16 * (st & 1);
-  #pragma unroll
+#pragma unroll
             for (int i = 0; i < 16; ++i) {
               const uint32_t xr = __shfl_sync(0xffffffffu, xrow_lane, i0 + i);
               if (row0 + i0 + i < M) {
