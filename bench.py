@@ -328,6 +328,10 @@ def run_ours(args, rank, world, local_rank):
                          None, stream.cuda_stream)
         torch.cuda.synchronize()
         segment["trace"] = b.sr_trace_read(senc.handle, reset=True)
+        # the two stream copies the timed forward also runs (widen x, narrow the
+        # output), from the traced steps, where each interval includes its launch
+        cp = segment["trace"].get("copy", {})
+        segment["copies_ms_traced"] = cp.get("ms", 0.0) / args.steps
         b.sr_trace_enable(senc.handle, False)
         senc.close()
 
@@ -569,8 +573,10 @@ def main():
         "sparse_segment": (dict(segment, frac_of_burst=segment["tflops"] / peaks["bf16_tflops"],
                                 frac_of_sustained=segment["tflops"] /
                                 peaks["bf16_tflops_sustained"],
-                                note="select + gather + the sparse blocks + delta scatter, "
-                                     "timed alone (split 0,n2,0), algorithmic flops of the "
+                                note="a forward of the n2 sparse blocks alone (split 0,n2,0): "
+                                     "select, gather, the sparse blocks and the delta scatter, "
+                                     "plus the widen of x to the fp32 stream and the narrow of "
+                                     "the output (copies_ms_traced); algorithmic flops of the "
                                      "sparse blocks")
                            if segment and wl.dtype == "bf16" else segment),
         "kernels": detail,
