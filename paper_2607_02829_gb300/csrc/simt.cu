@@ -8,7 +8,7 @@
 namespace sr {
 namespace {
 
-constexpr int BN = 64, BK = 16;
+constexpr int BN = 64, BK = 64;
 
 // Shared epilogue of every GEMM variant, applied to one output element.
 template <typename T, Epi E>
@@ -45,8 +45,9 @@ __device__ __forceinline__ float4 load4(const bf16* p) {
 
 // BM x 64 output tile per CTA of 256 threads (BM = 64 or 32: 4 or 2 rows x 4
 // columns per thread); the 32-row tile doubles the CTAs of small GEMMs.  The
-// next k-slice of A and W is loaded into registers (4 consecutive k per load)
-// while the current one is multiplied from shared memory.
+// next 64-column k-slice of A and W is loaded into registers (4 consecutive k
+// per load, 4 loads per matrix and thread) while the current one is multiplied
+// from shared memory.
 // kPart: split-K; CTA z of the grid's third dimension multiplies the K / gridDim.z
 // columns from z * K / gridDim.z on and stores its raw sums in part[z][M][N]
 // (the epilogue runs in splitk_epilogue_kernel).
@@ -63,22 +64,36 @@ gemm_simt_kernel(const T* __restrict__ A, const T* __restrict__ W, int M, int N,
   const int tx = tid & 15, ty = tid >> 4;
   const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
   float acc[RI][4] = {};
-  const int lr = tid >> 2, lk = (tid & 3) * 4;   // loader: row lr, k lk..lk+3
+  // loader: row lr, k lk + 16u .. lk + 16u + 3 for u = 0..3
+  constexpr int kLq = BK / 16;
+  const int lr = tid >> 2, lk = (tid & 3) * 4;
   const int am = m0 + lr, bn = n0 + lr;
   const bool a_ok = lr < BM && am < M, b_ok = bn < N;
   const T* ap = A + size_t(a_ok ? am : 0) * K + kz + lk;
   const T* bp = W + size_t(b_ok ? bn : 0) * K + kz + lk;
   const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
-  float4 ra = a_ok ? load4(ap) : zero, rb = b_ok ? load4(bp) : zero;
+  float4 ra[kLq], rb[kLq];
+#pragma unroll
+  for (int u = 0; u < kLq; ++u) {
+    ra[u] = a_ok ? load4(ap + 16 * u) : zero;
+    rb[u] = b_ok ? load4(bp + 16 * u) : zero;
+  }
   for (int k0 = 0; k0 < Kc; k0 += BK) {
-    if (lr < BM) {
-      As[lk][lr] = ra.x; As[lk + 1][lr] = ra.y; As[lk + 2][lr] = ra.z; As[lk + 3][lr] = ra.w;
+#pragma unroll
+    for (int u = 0; u < kLq; ++u) {
+      const int kk = lk + 16 * u;
+      if (lr < BM) {
+        As[kk][lr] = ra[u].x; As[kk + 1][lr] = ra[u].y; As[kk + 2][lr] = ra[u].z; As[kk + 3][lr] = ra[u].w;
+      }
+      Bs[kk][lr] = rb[u].x; Bs[kk + 1][lr] = rb[u].y; Bs[kk + 2][lr] = rb[u].z; Bs[kk + 3][lr] = rb[u].w;
     }
-    Bs[lk][lr] = rb.x; Bs[lk + 1][lr] = rb.y; Bs[lk + 2][lr] = rb.z; Bs[lk + 3][lr] = rb.w;
     __syncthreads();
     if (k0 + BK < Kc) {
-      ra = a_ok ? load4(ap + k0 + BK) : zero;
-      rb = b_ok ? load4(bp + k0 + BK) : zero;
+#pragma unroll
+      for (int u = 0; u < kLq; ++u) {
+        ra[u] = a_ok ? load4(ap + k0 + BK + 16 * u) : zero;
+        rb[u] = b_ok ? load4(bp + k0 + BK + 16 * u) : zero;
+      }
     }
 #pragma unroll
     for (int k = 0; k < BK; ++k) {
